@@ -1,0 +1,425 @@
+"""Benchmark of the geometric delta transport on GB300.
+
+One bench step = one pass of the whole hot path over a batch of assets:
+tau (per-asset tolerance), then a DDIM trajectory of S sampler steps in which
+the host picks full / cached and the rotating anchors, cached steps run the
+fused correspondence + delta transport + reconstruction kernel, and full
+steps run the passthrough reconstruction.  The denoiser's x0 outputs are
+seeded synthetic tensors already resident in HBM.
+
+value = target view-pixels transported + reconstructed per second, i.e.
+sum over cached steps of B * (N - a) * H * W, divided by the trajectory time.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+Under torchrun each rank runs its own batch of assets (weak scaling, no
+collective on the data path); rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "target view-pixels transported+reconstructed/sec per step; % of GB300 HBM BW"
+UNIT = "target view-pixels/s"
+L2_BYTES = 129 * 1024 * 1024
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--workload", default="batch128")
+    p.add_argument("--assets", type=int, default=64, help="assets per GPU (the batch128 sweep axis)")
+    p.add_argument("--corr", default="geometry", choices=["geometry", "table"])
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--cpu-assets", type=int, default=4, help="assets in the oracle's timed sample")
+    return p.parse_args()
+
+
+# ------------------------------------------------------------------ setup --
+def dist_env():
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    local = int(os.environ.get("LOCAL_RANK", 0))
+    return rank, world, local
+
+
+def workload(args, rank=0):
+    from paper_2608_13255_gb300 import synth
+    # each rank renders its own independent assets
+    base = synth.WORKLOADS[args.workload]
+    return synth.make_workload(args.workload, B=args.assets, seed=base["seed"] + 7919 * rank)
+
+
+def describe(w):
+    return ("%s: %d assets x %d views, %dx%dx%d %s latents + f32 x0 cache, %d rotating anchors, "
+            "%d-step %s, schedule %s, K=%d" % (w.name, w.B, w.N, w.H, w.W, w.C, w.dtype, w.a, w.S,
+                                              w.sampler.upper(), json.dumps(w.schedule), w.K))
+
+
+def step_bytes(w):
+    """Algorithmic HBM bytes of one cached transport step (latents only):
+    non-anchor element: x0_prev 4 + x0 write 4 + x_t 2 + x_next 2 (bf16) = 12 B;
+    anchor element: x0_new 4 + x0_prev 4 (for the increment) + cache write 4 + 4 (latents) = 16 B."""
+    lb = 2 if w.dtype == "bf16" else 4
+    hw = w.H * w.W
+    non = w.B * (w.N - w.a) * w.C * hw * (8 + 2 * lb)
+    anc = w.B * w.a * w.C * hw * (12 + 2 * lb)
+    return non + anc
+
+
+class Trajectory:
+    """Device state of one batch's trajectory and the loop over its steps."""
+
+    def __init__(self, w, dev, corr_mode="geometry"):
+        import torch
+        from paper_2608_13255_gb300 import geocache as gc
+        from paper_2608_13255_gb300 import synth
+        self.gc, self.w, self.dev = gc, w, dev
+        self.sched = w.schedule
+        self.pos = torch.from_numpy(w.pos).to(dev)
+        self.valid = torch.from_numpy(w.valid).to(dev)
+        self.cams = torch.from_numpy(w.cams).to(dev)
+        self.tau = torch.zeros(w.B, dtype=torch.float32, device=dev)
+        idx = wt = None
+        if corr_mode == "table":
+            shp = (w.B, w.N, w.N, w.H, w.W, w.K)
+            idx = torch.empty(shp, dtype=torch.int32, device=dev)
+            wt = torch.empty(shp, dtype=torch.float32, device=dev)
+        self.corr = gc.make_corr(self.pos, self.valid, self.cams, self.tau, idx, wt, K=w.K, tol_frac=w.tol_frac,
+                                 mode=gc.CORR_TABLE if corr_mode == "table" else gc.CORR_GEOMETRY)
+        xT, x0 = synth.initial_latents(w)
+        lat = torch.bfloat16 if w.dtype == "bf16" else torch.float32
+        self.x = torch.from_numpy(xT).to(dev).to(lat)
+        x0_d = torch.from_numpy(x0).to(dev)
+        self.full_x0, self.anchor_x0, self.recon = {}, {}, {}
+        for t in range(w.S):
+            p = synth.recon_params(w, t)
+            self.recon[t] = gc.make_recon(p["sampler"], a_t=p.get("a_t", 0), a_prev=p.get("a_prev", 0),
+                                          sigma=p.get("sigma", 0), sigma_next=p.get("sigma_next", 0))
+            anchors, full = gc.rotate_anchors(w.N, w.a, t, w.S, self.sched)
+            if full:
+                d = torch.from_numpy(synth.delta(w, t, list(range(w.N)))).to(dev)
+                self.full_x0[t] = (x0_d + d).contiguous()
+            else:
+                d = torch.from_numpy(synth.delta(w, t, anchors)).to(dev)
+                self.anchor_x0[t] = (x0_d[:, anchors] + d).contiguous()
+        self.bufs = [torch.empty_like(x0_d), torch.empty_like(x0_d)]
+        self.n_cached = len(self.anchor_x0)
+        self.pixels = self.n_cached * w.B * (w.N - w.a) * w.H * w.W
+
+    def host_inputs(self):
+        """Pinned host copies of every input of one trajectory (for e2e)."""
+        import torch
+        pin = lambda t: t.cpu().pin_memory()
+        return {"pos": pin(self.pos), "valid": pin(self.valid), "cams": pin(self.cams), "x": pin(self.x),
+                "full": {t: pin(v) for t, v in self.full_x0.items()},
+                "anchor": {t: pin(v) for t, v in self.anchor_x0.items()}}
+
+    def run(self, events=None):
+        """Enqueue one trajectory; returns the number of kernels launched.
+        events: list receiving (start, end) CUDA events around each cached-step launch."""
+        import torch
+        gc, w = self.gc, self.w
+        launches = 0
+        gc.build_corr(self.corr)
+        launches += 1 + (1 if self.corr.idx is not None else 0)
+        cache = None
+        for t in range(w.S):
+            anchors, full = gc.rotate_anchors(w.N, w.a, t, w.S, self.sched)
+            if full:
+                cache = self.full_x0[t]
+                gc.reconstruct(self.x, cache, self.x, self.recon[t])
+                launches += 1
+            else:
+                out = self.bufs[0] if cache is not self.bufs[0] else self.bufs[1]
+                if events is not None:
+                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    e0.record()
+                gc.transport_step(self.corr, anchors, w.C, self.anchor_x0[t], cache, out, self.x, self.x,
+                                  self.recon[t])
+                if events is not None:
+                    e1.record()
+                    events.append((e0, e1))
+                launches += (w.C + 15) // 16 if w.C > 4 else 1
+                cache = out
+        return launches
+
+    def run_e2e(self, host):
+        """One trajectory from pinned host inputs to a host copy of the final latents."""
+        import torch
+        self.pos.copy_(host["pos"], non_blocking=True)
+        self.valid.copy_(host["valid"], non_blocking=True)
+        self.cams.copy_(host["cams"], non_blocking=True)
+        self.x.copy_(host["x"], non_blocking=True)
+        for t, v in host["full"].items():
+            self.full_x0[t].copy_(v, non_blocking=True)
+        for t, v in host["anchor"].items():
+            self.anchor_x0[t].copy_(v, non_blocking=True)
+        self.run()
+        out = torch.empty(self.x.shape, dtype=self.x.dtype, pin_memory=True)
+        out.copy_(self.x, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+        return out
+
+    def h2d_bytes(self):
+        n = lambda t: t.numel() * t.element_size()
+        return (n(self.pos) + n(self.valid) + n(self.cams) + n(self.x) + sum(n(v) for v in self.full_x0.values())
+                + sum(n(v) for v in self.anchor_x0.values()))
+
+    def working_set(self):
+        n = lambda t: t.numel() * t.element_size()
+        return 2 * n(self.x) + 2 * n(self.bufs[0]) + n(next(iter(self.anchor_x0.values())))
+
+
+# ----------------------------------------------------------------- clocks --
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", "clocks_rank%d.csv" % gpu_index)
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+# ------------------------------------------------------------ CPU oracle --
+def oracle_trajectory(w, steps=None):
+    """The CPU oracle, as it stands, over one trajectory of workload w.
+    Returns (cached target view-pixels processed, seconds)."""
+    import oracle
+    from paper_2608_13255_gb300 import synth
+    t0 = time.perf_counter()
+    tau = oracle.tau(w.pos, w.valid, w.tol_frac)
+    geom = (w.pos, w.valid, w.cams, tau)
+    xT, x0 = synth.initial_latents(w)
+    x = xT.astype(np.float64)
+    cache = x0.astype(np.float64)
+    pixels = 0
+    S = w.S if steps is None else steps
+    for t in range(S):
+        p = synth.recon_params(w, t)
+        rk = dict(sampler=oracle.DDIM if p["sampler"] == "ddim" else oracle.FM_EULER, a_t=p.get("a_t", 0.0),
+                  a_prev=p.get("a_prev", 0.0), sigma=p.get("sigma", 0.0), sigma_next=p.get("sigma_next", 0.0))
+        if oracle.is_full_step(t, w.S, w.schedule):
+            cache = cache + synth.delta(w, t, list(range(w.N)))
+            x, _ = oracle.reconstruct(x, cache, **rk)
+        else:
+            anchors = oracle.rotate_anchors(w.N, w.a, oracle.cached_ordinal(t, w.S, w.schedule))
+            new = cache[:, anchors] + synth.delta(w, t, anchors)
+            cache, x, _ = oracle.transport_step(anchors, new, cache, geom=geom, x_t=x, recon=rk)
+            pixels += w.B * (w.N - w.a) * w.H * w.W
+        if w.dtype == "bf16":
+            x = (oracle.round_bf16(x).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return pixels, time.perf_counter() - t0
+
+
+def cpu_baseline(args, w_full):
+    from paper_2608_13255_gb300 import synth
+    ws = synth.replicate_assets(w_full, args.cpu_assets)
+    pixels, secs = oracle_trajectory(ws)
+    return {"value": pixels / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": "%d of the %d assets, one whole %d-step trajectory (%.1f s, single-threaded C oracle)" % (
+                args.cpu_assets, w_full.B, w_full.S, secs)}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2608_13255_gb300 import synth
+    w = workload(args)
+    ws = synth.replicate_assets(w, args.cpu_assets)
+    for _ in range(args.warmup):
+        oracle_trajectory(ws, steps=6)
+    tot_pix, tot_s = 0, 0.0
+    for _ in range(args.steps):
+        pix, s = oracle_trajectory(ws)
+        tot_pix += pix
+        tot_s += s
+    value = tot_pix / tot_s
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": describe(w), "sampled_assets": args.cpu_assets},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": "%d of %d assets per step, whole trajectories" % (args.cpu_assets, w.B)},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+# ------------------------------------------------------------------- main --
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import torch
+    import torch.distributed as dist
+    rank, world, local = dist_env()
+    if world > 1:
+        dist.init_process_group("gloo")
+    torch.cuda.set_device(local)
+    dev = "cuda:%d" % local
+    from paper_2608_13255_gb300 import build as gbuild
+    gbuild.build()
+    w = workload(args, rank)
+    traj = Trajectory(w, dev, args.corr)
+    ws_bytes = traj.working_set()
+
+    args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
+    for _ in range(args.warmup):
+        traj.run()
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    events = []
+    launches = 0
+    with ClockSampler(local) as clocks:
+        barrier()
+        torch.cuda.synchronize()
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for _ in range(args.steps):
+            launches += traj.run(events)
+        t1.record()
+        torch.cuda.synchronize()
+        barrier()
+    ms = t0.elapsed_time(t1)
+    kernel_ms = [a.elapsed_time(b) for a, b in events]
+    if world > 1:
+        tt = torch.tensor([ms], dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms = float(tt.item())
+    ms_per_step = ms / args.steps
+    total_pixels = traj.pixels * world
+    value = total_pixels / (ms_per_step / 1e3)
+
+    k_avg_ms = sum(kernel_ms) / len(kernel_ms)
+    alg = step_bytes(w)
+    achieved = alg / (k_avg_ms / 1e3) / 1e9
+    peak, peak_src = measured_peak()
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "transport_traffic.json")
+    if os.path.exists(tpath):
+        try:
+            tj = json.load(open(tpath))
+            if tj.get("kernel_hash") == gbuild.source_hash() and tj.get("assets") and tj.get("bytes"):
+                traffic = tj["bytes"] * (w.B / tj["assets"])
+        except (OSError, ValueError):
+            traffic = None
+
+    e2e = None
+    if not args.no_e2e:
+        host = traj.host_inputs()
+        traj.run_e2e(host)
+        barrier()
+        t_s = time.perf_counter()
+        for _ in range(args.steps):
+            out = traj.run_e2e(host)
+        e2e_s = (time.perf_counter() - t_s) / args.steps
+        if world > 1:
+            tt = torch.tensor([e2e_s], dtype=torch.float64)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e2e_s = float(tt.item())
+        e2e = {"value": total_pixels / e2e_s, "unit": UNIT, "h2d_bytes_per_step": traj.h2d_bytes(),
+               "d2h_bytes_per_step": out.numel() * out.element_size(), "ms_per_step": 1e3 * e2e_s}
+
+    if rank != 0:
+        return 0
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": describe(w), "assets_per_gpu": w.B, "corr": args.corr,
+                   "storage": "bf16 latents, f32 x0 cache" if w.dtype == "bf16" else "f32",
+                   "l2": "inputs larger than L2: %.0f MB touched per cached step vs %d MB L2" % (
+                       ws_bytes / 1e6, L2_BYTES // 2 ** 20),
+                   "step": "tau + %d-step trajectory (%d cached transport steps, %d full steps)" % (
+                       w.S, traj.n_cached, w.S - traj.n_cached)},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
+                     "kernel": "transport_kernel", "alg_bytes_per_launch": alg,
+                     "avg_launch_us": 1e3 * k_avg_ms, "launches": len(kernel_ms),
+                     "frac_of_8TBs": achieved / 8000.0},
+        "gpu_launches": launches,
+        "clocks": clocks.summary(),
+        "e2e": e2e,
+    }
+    if not args.no_cpu and world == 1:
+        line["cpu_baseline"] = cpu_baseline(args, w)
+    print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,223 @@
+/*
+ * geocache.h -- C ABI of libgeocache.so: geometric delta transport between the
+ * views of a multi-view diffusion batch (GeoCache, Sec. 3.2 of the paper),
+ * computed by CUDA kernels for sm_103a on one GPU.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Pointers marked "device" are CUDA device addresses on the current device
+ *   (e.g. torch tensors' data_ptr()); pointers marked "host" are ordinary host
+ *   memory.  The caller owns every buffer; the library keeps no device state
+ *   between calls and allocates no memory.
+ * - Every device-side entry point is asynchronous on `stream` (a cudaStream_t,
+ *   NULL = the legacy default stream) and returns after enqueueing its kernels.
+ * - Latents are NCHW per view with the views on the batch axis:
+ *   [B, N, C, H, W] contiguous (B assets, N views, C channels, H x W tokens).
+ *   Position maps and correspondence tables use the same token grid.
+ * - Arguments are checked before anything is launched; a non-OK status means
+ *   nothing was enqueued (except GEOCACHE_ECUDA, which reports a launch
+ *   failure after enqueueing) and geocache_last_error() describes the problem.
+ */
+#ifndef GEOCACHE_H
+#define GEOCACHE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define GEOCACHE_ABI_VERSION 1
+#define GEOCACHE_MAX_VIEWS 64   /* N <= 64 */
+#define GEOCACHE_MAX_CHANNELS 1024
+
+typedef enum {
+    GEOCACHE_OK = 0,
+    GEOCACHE_EINVAL = -1,   /* NULL pointer, bad enum, bad anchors, bad sampler parameters */
+    GEOCACHE_ESHAPE = -2,   /* a size is out of range */
+    GEOCACHE_EDTYPE = -3,   /* unsupported latent dtype */
+    GEOCACHE_ECUDA = -4,    /* a CUDA call or kernel launch failed */
+    GEOCACHE_ETIMEOUT = -5, /* reserved: a bounded device wait gave up */
+    GEOCACHE_EDEVICE = -6,  /* no usable CUDA device */
+    GEOCACHE_EALIAS = -7    /* buffers overlap in a way the call does not allow */
+} geocache_status;
+
+typedef enum { GEOCACHE_F32 = 0, GEOCACHE_BF16 = 1 } geocache_dtype;
+
+typedef enum { GEOCACHE_DDIM = 0, GEOCACHE_FM_EULER = 1 } geocache_sampler;
+
+/* Optional per-element prediction written next to x_{t-1}: the quantity a
+ * sampler keeps in its history (Sec. 3.2, closed-form conversion after Eq. 1). */
+typedef enum {
+    GEOCACHE_PRED_NONE = 0,
+    GEOCACHE_PRED_EPS = 1,      /* DDIM: eps = (x_t - sqrt(ab_t) x0) / sqrt(1 - ab_t) */
+    GEOCACHE_PRED_V = 2,        /* DDIM: v = sqrt(ab_t) eps - sqrt(1 - ab_t) x0 */
+    GEOCACHE_PRED_VELOCITY = 3  /* FM: u = (x_sigma - x0) / sigma */
+} geocache_pred;
+
+/* How geocache_transport_step obtains the taps of G_{u->v}. */
+typedef enum {
+    GEOCACHE_CORR_GEOMETRY = 0, /* recompute them from pos/valid/cams/tau (bit-identical to the tables) */
+    GEOCACHE_CORR_TABLE = 1     /* read idx/w written by geocache_build_corr (or supplied by the caller) */
+} geocache_corr_mode;
+
+/* Pinhole camera, world -> camera: x_c = R x_w + t (R row-major), +z forward,
+ * pixel x right, pixel y down, token (i, j) centred at (i + 0.5, j + 0.5).
+ * 64 bytes. */
+typedef struct {
+    float R[9];
+    float t[3];
+    float fx, fy, cx, cy;
+} geocache_camera;
+
+/* Correspondence operator G_{u->v} of one batch of assets (Sec. 3.2,
+ * "Correspondence operator"): for target token p of view v, the K taps of
+ * source view u around the projection of X = P_v(p) whose 3-D positions lie
+ * within tau of X, with area (bilinear) weights renormalised to sum to one;
+ * rows without a kept tap are zero.  K = 4 (bilinear footprint) or K = 1
+ * (the token containing the projection).
+ * tau = tol_frac * diagonal of the box of the asset's foreground texels
+ * (tol_frac = 0.01 in the paper).
+ * The struct only records caller-owned device buffers; they must stay valid
+ * while calls use the struct. */
+typedef struct {
+    int B, N, H, W, K;
+    float tol_frac;
+    const float* pos;               /* device [B,N,H,W,3] f32 world positions of each token */
+    const uint8_t* valid;           /* device [B,N,H,W] u8, nonzero = foreground */
+    const geocache_camera* cams;    /* device [B,N] */
+    float* tau;                     /* device [B] f32, written by geocache_build_corr */
+    int32_t* idx;                   /* device [B,N(v),N(u),H,W,K] i32 source token index row*W+col,
+                                       -1 = tap not kept; or NULL (tables not built) */
+    float* w;                       /* device [B,N(v),N(u),H,W,K] f32 weights, 0 where idx = -1; or NULL */
+    geocache_corr_mode mode;        /* taps used by geocache_transport_step */
+} geocache_corr;
+
+/* Sampler step parameters (Sec. 3.2, closed-form conversion after Eq. 1).
+ * DDIM (eta = 0): 0 < a_t < 1 and 0 < a_prev <= 1 are alpha-bar at this step
+ * and at the next one:
+ *     eps = (x_t - sqrt(a_t) x0) / sqrt(1 - a_t),
+ *     x_next = sqrt(a_prev) x0 + sqrt(1 - a_prev) eps.
+ * Flow-matching Euler (x_s = (1 - s) x0 + s eps): sigma > 0, sigma_next >= 0:
+ *     u = (x_s - x0) / sigma,  x_next = x_s + (sigma_next - sigma) u.
+ * The square roots and reciprocals are formed once in double on the host and
+ * rounded to float; the per-element arithmetic is float. */
+typedef struct {
+    geocache_sampler sampler;
+    double a_t, a_prev;
+    double sigma, sigma_next;
+    geocache_pred pred_kind;
+    float* pred_out;   /* device f32, same shape as x_next, or NULL (pred_kind must then be NONE) */
+} geocache_recon;
+
+/* Full / cached step policy (Sec. 3.2, drift-bounding schedule). Step 0 is
+ * always full (no x0(t-1) exists) except under SINGLE_CACHED. */
+typedef enum {
+    GEOCACHE_SCHED_EVERY_K = 0,       /* full iff step % k == 0 */
+    GEOCACHE_SCHED_HEAD_MID_TAIL = 1, /* first `head` steps, step S/2 if mid != 0, last `tail` steps */
+    GEOCACHE_SCHED_LIST = 2,          /* full iff step is in full_steps[0..n_full_steps) */
+    GEOCACHE_SCHED_ALL_FULL = 3,      /* every step full (the a = N gate) */
+    GEOCACHE_SCHED_SINGLE_CACHED = 4  /* step 0 is a supplied state; every later step is cached */
+} geocache_sched_kind;
+
+typedef struct {
+    geocache_sched_kind kind;
+    int k;
+    int head, mid, tail;
+    const int32_t* full_steps;        /* host, for GEOCACHE_SCHED_LIST */
+    int n_full_steps;
+    int contiguous_rotation;          /* 0: strided rotation (default), 1: contiguous blocks */
+} geocache_schedule;
+
+/* --------------------------------------------------------------------------
+ * geocache_build_corr -- tau and the correspondence tables (Sec. 3.2,
+ * "Correspondence operator"; precomputed once per asset).
+ *
+ * Reads corr->pos, corr->valid, corr->cams; writes corr->tau[B] and, when
+ * corr->idx and corr->w are both non-NULL, the tables for every ordered pair
+ * (v, u): the diagonal u == v and background targets hold idx -1 / w 0.
+ * Sizes: 1 <= B, 2 <= N <= GEOCACHE_MAX_VIEWS, 1 <= H, W <= 16384,
+ * K in {1, 4}, 0 < tol_frac.  tau must not overlap the other buffers.
+ * Returns GEOCACHE_OK, EINVAL (NULL / bad K / tol_frac), ESHAPE, ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_build_corr(geocache_corr* corr, void* stream);
+
+/* --------------------------------------------------------------------------
+ * geocache_transport_step -- one cached sampler step (Eq. 1 and the
+ * multi-anchor aggregation, invalid-match and loop-order paragraphs of
+ * Sec. 3.2), fused with the sampler reconstruction when recon != NULL.
+ *
+ *   anchors   host [a], ascending, distinct, in [0, N): the views the
+ *             denoiser ran on at this step (1 <= a <= N).
+ *   x0_anchor_new  device [B,a,C,H,W] f32: the denoiser's x0 for the anchors,
+ *             in the order of `anchors`.
+ *   x0_prev   device [B,N,C,H,W] f32: stored x0(t-1) of every view.
+ *   x0_out    device [B,N,C,H,W] f32: receives x0(t) of every view:
+ *             anchors: x0_anchor_new; other views v:
+ *               x0_prev^v + (1/n) sum_{u in A with a kept tap} sum_k w_k Delta^u[q_k],
+ *             Delta^u = x0_anchor_new^u - x0_prev^u, n = number of such u;
+ *             n = 0 keeps x0_prev^v.
+ *             x0_out may equal x0_prev (in-place update; the anchors' rows are
+ *             then written by a second kernel after the gathers) but must not
+ *             otherwise overlap it.
+ *   x_t, x_next  device [B,N,C,H,W] of lat_dtype (F32 or BF16): when recon is
+ *             non-NULL, x_next = reconstruction of x_t with x0(t) for every
+ *             view (bf16 stores round to nearest even); x_next may equal x_t.
+ *             Ignored when recon is NULL.
+ *   C         1 <= C <= GEOCACHE_MAX_CHANNELS.
+ * corr must have been filled by geocache_build_corr (tau, and idx/w in
+ * GEOCACHE_CORR_TABLE mode).
+ * Returns GEOCACHE_OK, EINVAL, ESHAPE, EDTYPE, EALIAS, ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_transport_step(const geocache_corr* corr, const int32_t* anchors, int a, int C,
+                            const float* x0_anchor_new, const float* x0_prev, float* x0_out,
+                            const void* x_t, void* x_next, geocache_dtype lat_dtype,
+                            const geocache_recon* recon, void* stream);
+
+/* --------------------------------------------------------------------------
+ * geocache_reconstruct -- full-step passthrough (Sec. 3.2: at a full step the
+ * denoiser runs on all N views and its x0 is both the new reference and the
+ * input of the sampler conversion).
+ *
+ *   x_t, x_next  device [n] of lat_dtype (may be equal);  x0 device [n] f32;
+ *   x0_store     device [n] f32 copy of x0 (the stored reference), or NULL.
+ * Returns GEOCACHE_OK, EINVAL, ESHAPE (n < 0), EDTYPE, EALIAS, ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_reconstruct(const void* x_t, const float* x0, void* x_next, geocache_dtype lat_dtype,
+                         int64_t n, const geocache_recon* recon, float* x0_store, void* stream);
+
+/* --------------------------------------------------------------------------
+ * geocache_is_full_step -- 1 if `step` (0 <= step < S) is a full step under
+ * `sched`, 0 if cached, a negative status on bad arguments. Host only.
+ * ------------------------------------------------------------------------ */
+int geocache_is_full_step(int step, int S, const geocache_schedule* sched);
+
+/* --------------------------------------------------------------------------
+ * geocache_rotate_anchors -- anchor set of `step` (Sec. 3.2, batch-sliced
+ * anchor forward: the anchors rotate every step and every view returns to the
+ * full context every ceil(N/a) steps).  Host only.
+ *
+ * With r = number of cached steps before `step` under `sched`:
+ *   strided (default): s = ceil(N/a), A = {(r mod s + j s) mod N : j < a};
+ *   contiguous:        A = {(r a + j) mod N : j < a};
+ * a repeated id is replaced by the smallest id not used by A otherwise.
+ * anchors_out (host [a]) receives A in ascending order; *is_full_out (may be
+ * NULL) receives 1 if the step is a full step (the anchors are then the ones
+ * the next cached step will use) and 0 otherwise.
+ * Returns GEOCACHE_OK, EINVAL, ESHAPE.
+ * ------------------------------------------------------------------------ */
+int geocache_rotate_anchors(int N, int a, int step, int S, const geocache_schedule* sched,
+                            int32_t* anchors_out, int* is_full_out);
+
+/* Thread-local description of the last non-OK status of this thread ("" if
+ * none).  The pointer stays valid until the thread's next library call. */
+const char* geocache_last_error(void);
+
+/* GEOCACHE_ABI_VERSION of the loaded library. */
+int geocache_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GEOCACHE_H */

@@ -1,0 +1,307 @@
+// C ABI of libgeocache.so (include/geocache.h): argument checking, the host
+// side of the anchor rotation and the refresh schedule, sampler constants,
+// and kernel launches.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdint>
+#include <cstdio>
+#include <string>
+
+#include "geocache.h"
+#include "geocache_internal.h"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int fail(int status, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return status;
+}
+
+int ok() {
+    g_last_error.clear();
+    return GEOCACHE_OK;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+    return fail(GEOCACHE_ECUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+// [a, a+na) and [b, b+nb) in bytes overlap
+bool overlap(const void* a, size_t na, const void* b, size_t nb) {
+    if (!a || !b || na == 0 || nb == 0) return false;
+    const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+    return x < y + nb && y < x + na;
+}
+
+int check_sizes(int B, int N, int H, int W) {
+    if (B < 1 || B > 65535) return fail(GEOCACHE_ESHAPE, "B=%d out of range [1, 65535]", B);
+    if (N < 2 || N > GEOCACHE_MAX_VIEWS) return fail(GEOCACHE_ESHAPE, "N=%d out of range [2, %d]", N, GEOCACHE_MAX_VIEWS);
+    if (H < 1 || W < 1 || H > 16384 || W > 16384) return fail(GEOCACHE_ESHAPE, "H=%d, W=%d out of range [1, 16384]", H, W);
+    return GEOCACHE_OK;
+}
+
+int make_coef(const geocache_recon* r, geocache::ReconCoef* c) {
+    *c = geocache::ReconCoef{};
+    if (!r) return GEOCACHE_OK;
+    c->enabled = 1;
+    c->sampler = r->sampler;
+    c->pred_kind = r->pred_kind;
+    if (r->pred_kind != GEOCACHE_PRED_NONE && !r->pred_out)
+        return fail(GEOCACHE_EINVAL, "pred_kind %d requires pred_out", (int)r->pred_kind);
+    if (r->pred_kind == GEOCACHE_PRED_NONE && r->pred_out)
+        return fail(GEOCACHE_EINVAL, "pred_out given with pred_kind NONE");
+    if (r->sampler == GEOCACHE_DDIM) {
+        if (!(r->a_t > 0.0 && r->a_t < 1.0)) return fail(GEOCACHE_EINVAL, "DDIM needs 0 < a_t < 1 (got %g)", r->a_t);
+        if (!(r->a_prev > 0.0 && r->a_prev <= 1.0))
+            return fail(GEOCACHE_EINVAL, "DDIM needs 0 < a_prev <= 1 (got %g)", r->a_prev);
+        if (r->pred_kind != GEOCACHE_PRED_NONE && r->pred_kind != GEOCACHE_PRED_EPS && r->pred_kind != GEOCACHE_PRED_V)
+            return fail(GEOCACHE_EINVAL, "DDIM prediction must be NONE, EPS or V");
+        c->st = (float)std::sqrt(r->a_t);
+        c->s1t = (float)std::sqrt(1.0 - r->a_t);
+        c->inv_s1t = (float)(1.0 / std::sqrt(1.0 - r->a_t));
+        c->sp = (float)std::sqrt(r->a_prev);
+        c->s1p = (float)std::sqrt(1.0 - r->a_prev);
+    } else if (r->sampler == GEOCACHE_FM_EULER) {
+        if (!(r->sigma > 0.0 && std::isfinite(r->sigma)))
+            return fail(GEOCACHE_EINVAL, "flow matching needs sigma > 0 (got %g)", r->sigma);
+        if (!(r->sigma_next >= 0.0 && std::isfinite(r->sigma_next)))
+            return fail(GEOCACHE_EINVAL, "flow matching needs sigma_next >= 0 (got %g)", r->sigma_next);
+        if (r->pred_kind != GEOCACHE_PRED_NONE && r->pred_kind != GEOCACHE_PRED_VELOCITY)
+            return fail(GEOCACHE_EINVAL, "flow-matching prediction must be NONE or VELOCITY");
+        c->inv_sigma = (float)(1.0 / r->sigma);
+        c->dsigma = (float)(r->sigma_next - r->sigma);
+    } else {
+        return fail(GEOCACHE_EINVAL, "unknown sampler %d", (int)r->sampler);
+    }
+    return GEOCACHE_OK;
+}
+
+size_t lat_bytes(int dtype) { return dtype == GEOCACHE_BF16 ? 2 : 4; }
+
+}  // namespace
+
+extern "C" {
+
+int geocache_abi_version(void) { return GEOCACHE_ABI_VERSION; }
+
+const char* geocache_last_error(void) { return g_last_error.c_str(); }
+
+int geocache_build_corr(geocache_corr* c, void* stream) {
+    if (!c) return fail(GEOCACHE_EINVAL, "corr is NULL");
+    int st = check_sizes(c->B, c->N, c->H, c->W);
+    if (st) return st;
+    if (c->K != 1 && c->K != 4) return fail(GEOCACHE_EINVAL, "K=%d must be 1 or 4", c->K);
+    if (!(c->tol_frac > 0.0f) || !std::isfinite(c->tol_frac))
+        return fail(GEOCACHE_EINVAL, "tol_frac=%g must be positive", (double)c->tol_frac);
+    if (!c->pos || !c->valid || !c->cams || !c->tau) return fail(GEOCACHE_EINVAL, "pos, valid, cams and tau are required");
+    if ((c->idx == nullptr) != (c->w == nullptr)) return fail(GEOCACHE_EINVAL, "idx and w must both be given or both NULL");
+    const size_t texels = (size_t)c->B * c->N * c->H * c->W;
+    if (overlap(c->tau, sizeof(float) * c->B, c->pos, texels * 12) ||
+        overlap(c->tau, sizeof(float) * c->B, c->valid, texels) ||
+        overlap(c->tau, sizeof(float) * c->B, c->cams, sizeof(geocache_camera) * c->B * c->N))
+        return fail(GEOCACHE_EALIAS, "tau overlaps an input");
+    if (c->idx) {
+        const size_t rows = texels * c->N * c->K;
+        if (c->K == 4 && (((uintptr_t)c->idx | (uintptr_t)c->w) & 15))
+            return fail(GEOCACHE_EINVAL, "idx and w must be 16-byte aligned for K=4");
+        if (overlap(c->idx, rows * 4, c->w, rows * 4)) return fail(GEOCACHE_EALIAS, "idx and w overlap");
+    }
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e = geocache::launch_tau(c->pos, c->valid, c->B, c->N, c->H, c->W, c->tol_frac, c->tau, s);
+    if (e != cudaSuccess) return cuda_fail(e, "tau kernel launch");
+    if (c->idx) {
+        e = geocache::launch_build_corr(*c, s);
+        if (e != cudaSuccess) return cuda_fail(e, "correspondence kernel launch");
+    }
+    return ok();
+}
+
+int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int a, int C,
+                            const float* x0_anchor_new, const float* x0_prev, float* x0_out, const void* x_t,
+                            void* x_next, geocache_dtype lat_dtype, const geocache_recon* recon, void* stream) {
+    if (!c) return fail(GEOCACHE_EINVAL, "corr is NULL");
+    int st = check_sizes(c->B, c->N, c->H, c->W);
+    if (st) return st;
+    if (c->K != 1 && c->K != 4) return fail(GEOCACHE_EINVAL, "K=%d must be 1 or 4", c->K);
+    if (C < 1 || C > GEOCACHE_MAX_CHANNELS) return fail(GEOCACHE_ESHAPE, "C=%d out of range [1, %d]", C, GEOCACHE_MAX_CHANNELS);
+    if (c->mode == GEOCACHE_CORR_GEOMETRY) {
+        if (!c->pos || !c->valid || !c->cams || !c->tau)
+            return fail(GEOCACHE_EINVAL, "geometry mode needs pos, valid, cams and tau");
+    } else if (c->mode == GEOCACHE_CORR_TABLE) {
+        if (!c->idx || !c->w) return fail(GEOCACHE_EINVAL, "table mode needs idx and w");
+    } else {
+        return fail(GEOCACHE_EINVAL, "unknown corr mode %d", (int)c->mode);
+    }
+    if (!anchors) return fail(GEOCACHE_EINVAL, "anchors is NULL");
+    if (a < 1 || a > c->N) return fail(GEOCACHE_EINVAL, "a=%d must be in [1, N=%d]", a, c->N);
+    for (int s = 0; s < a; ++s) {
+        if (anchors[s] < 0 || anchors[s] >= c->N) return fail(GEOCACHE_EINVAL, "anchor %d out of range", anchors[s]);
+        if (s && anchors[s] <= anchors[s - 1]) return fail(GEOCACHE_EINVAL, "anchors must be ascending and distinct");
+    }
+    if (!x0_anchor_new || !x0_prev || !x0_out) return fail(GEOCACHE_EINVAL, "x0 buffers are required");
+    if (lat_dtype != GEOCACHE_F32 && lat_dtype != GEOCACHE_BF16)
+        return fail(GEOCACHE_EDTYPE, "unsupported latent dtype %d", (int)lat_dtype);
+    geocache::ReconCoef coef;
+    st = make_coef(recon, &coef);
+    if (st) return st;
+    const size_t HW = (size_t)c->H * c->W;
+    const size_t n_all = (size_t)c->B * c->N * C * HW, n_anc = (size_t)c->B * a * C * HW;
+    if (recon && (!x_t || !x_next)) return fail(GEOCACHE_EINVAL, "reconstruction needs x_t and x_next");
+    if (x0_out != x0_prev && overlap(x0_out, n_all * 4, x0_prev, n_all * 4))
+        return fail(GEOCACHE_EALIAS, "x0_out partially overlaps x0_prev");
+    if (overlap(x0_out, n_all * 4, x0_anchor_new, n_anc * 4)) return fail(GEOCACHE_EALIAS, "x0_out overlaps x0_anchor_new");
+    if (recon) {
+        const size_t lb = lat_bytes(lat_dtype);
+        if (x_next != x_t && overlap(x_next, n_all * lb, x_t, n_all * lb))
+            return fail(GEOCACHE_EALIAS, "x_next partially overlaps x_t");
+        if (overlap(x_next, n_all * lb, x0_out, n_all * 4) || overlap(x_next, n_all * lb, x0_prev, n_all * 4) ||
+            overlap(x_next, n_all * lb, x0_anchor_new, n_anc * 4))
+            return fail(GEOCACHE_EALIAS, "x_next overlaps an x0 buffer");
+        if (recon->pred_out &&
+            (overlap(recon->pred_out, n_all * 4, x0_out, n_all * 4) || overlap(recon->pred_out, n_all * 4, x_next, n_all * lb) ||
+             overlap(recon->pred_out, n_all * 4, x0_prev, n_all * 4) || overlap(recon->pred_out, n_all * 4, x_t, n_all * lb)))
+            return fail(GEOCACHE_EALIAS, "pred_out overlaps another buffer");
+    }
+    geocache::TransportArgs t{};
+    t.B = c->B; t.N = c->N; t.H = c->H; t.W = c->W; t.C = C; t.K = c->K; t.a = a;
+    t.mode = c->mode;
+    t.write_anchor_rows = (x0_out != x0_prev);
+    t.lat_dtype = lat_dtype;
+    t.pos = c->pos; t.valid = c->valid; t.cams = c->cams; t.tau = c->tau; t.idx = c->idx; t.w = c->w;
+    t.x0_new = x0_anchor_new; t.x0_prev = x0_prev; t.x0_out = x0_out;
+    t.x_t = x_t; t.x_next = x_next; t.pred_out = recon ? recon->pred_out : nullptr;
+    t.coef = coef;
+    for (int v = 0; v < GEOCACHE_MAX_VIEWS; ++v) { t.slot_of[v] = -1; t.anchors[v] = -1; }
+    for (int s = 0; s < a; ++s) { t.anchors[s] = anchors[s]; t.slot_of[anchors[s]] = s; }
+    cudaStream_t s = (cudaStream_t)stream;
+    const int chunk = C <= 4 ? 4 : 16;
+    for (int c0 = 0; c0 < C; c0 += chunk) {
+        t.c0 = c0;
+        t.cn = C - c0 < chunk ? C - c0 : chunk;
+        cudaError_t e = geocache::launch_transport(t, s);
+        if (e != cudaSuccess) return cuda_fail(e, "transport kernel launch");
+    }
+    if (!t.write_anchor_rows) {
+        t.c0 = 0;
+        t.cn = C;
+        cudaError_t e = geocache::launch_copy_anchor_rows(t, s);
+        if (e != cudaSuccess) return cuda_fail(e, "anchor-row copy launch");
+    }
+    return ok();
+}
+
+int geocache_reconstruct(const void* x_t, const float* x0, void* x_next, geocache_dtype lat_dtype, int64_t n,
+                         const geocache_recon* recon, float* x0_store, void* stream) {
+    if (n < 0) return fail(GEOCACHE_ESHAPE, "n=%lld is negative", (long long)n);
+    if (!recon) return fail(GEOCACHE_EINVAL, "recon is NULL");
+    if (lat_dtype != GEOCACHE_F32 && lat_dtype != GEOCACHE_BF16)
+        return fail(GEOCACHE_EDTYPE, "unsupported latent dtype %d", (int)lat_dtype);
+    if (n > 0 && (!x_t || !x0 || !x_next)) return fail(GEOCACHE_EINVAL, "x_t, x0 and x_next are required");
+    geocache::ReconCoef coef;
+    int st = make_coef(recon, &coef);
+    if (st) return st;
+    const size_t lb = lat_bytes(lat_dtype), un = (size_t)n;
+    if (x_next != x_t && overlap(x_next, un * lb, x_t, un * lb))
+        return fail(GEOCACHE_EALIAS, "x_next partially overlaps x_t");
+    if (overlap(x_next, un * lb, x0, un * 4)) return fail(GEOCACHE_EALIAS, "x_next overlaps x0");
+    if (x0_store && x0_store != x0 &&
+        (overlap(x0_store, un * 4, x0, un * 4) || overlap(x0_store, un * 4, x_next, un * lb) ||
+         overlap(x0_store, un * 4, x_t, un * lb)))
+        return fail(GEOCACHE_EALIAS, "x0_store overlaps another buffer");
+    if (recon->pred_out && (overlap(recon->pred_out, un * 4, x_next, un * lb) || overlap(recon->pred_out, un * 4, x0, un * 4) ||
+                            overlap(recon->pred_out, un * 4, x_t, un * lb)))
+        return fail(GEOCACHE_EALIAS, "pred_out overlaps another buffer");
+    cudaError_t e = geocache::launch_reconstruct(x_t, x0, x_next, lat_dtype, n, coef, recon->pred_out,
+                                                 x0_store == x0 ? nullptr : x0_store, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "reconstruction kernel launch");
+    return ok();
+}
+
+int geocache_is_full_step(int step, int S, const geocache_schedule* sched) {
+    if (!sched) return fail(GEOCACHE_EINVAL, "schedule is NULL");
+    if (S < 1 || step < 0 || step >= S) return fail(GEOCACHE_ESHAPE, "step=%d outside [0, S=%d)", step, S);
+    switch (sched->kind) {
+        case GEOCACHE_SCHED_SINGLE_CACHED:
+            g_last_error.clear();
+            return step == 0 ? 1 : 0;
+        case GEOCACHE_SCHED_EVERY_K:
+            if (sched->k < 1) return fail(GEOCACHE_EINVAL, "every-k schedule needs k >= 1");
+            g_last_error.clear();
+            return step % sched->k == 0 ? 1 : 0;
+        case GEOCACHE_SCHED_HEAD_MID_TAIL:
+            if (sched->head < 0 || sched->tail < 0) return fail(GEOCACHE_EINVAL, "head and tail must be >= 0");
+            g_last_error.clear();
+            if (step == 0 || step < sched->head) return 1;
+            if (sched->mid && step == S / 2) return 1;
+            return step >= S - sched->tail ? 1 : 0;
+        case GEOCACHE_SCHED_LIST:
+            if (sched->n_full_steps < 0 || (sched->n_full_steps > 0 && !sched->full_steps))
+                return fail(GEOCACHE_EINVAL, "list schedule needs full_steps");
+            g_last_error.clear();
+            if (step == 0) return 1;
+            for (int i = 0; i < sched->n_full_steps; ++i)
+                if (sched->full_steps[i] == step) return 1;
+            return 0;
+        case GEOCACHE_SCHED_ALL_FULL:
+            g_last_error.clear();
+            return 1;
+    }
+    return fail(GEOCACHE_EINVAL, "unknown schedule kind %d", (int)sched->kind);
+}
+
+int geocache_rotate_anchors(int N, int a, int step, int S, const geocache_schedule* sched, int32_t* anchors_out,
+                            int* is_full_out) {
+    if (!anchors_out) return fail(GEOCACHE_EINVAL, "anchors_out is NULL");
+    if (N < 1 || N > GEOCACHE_MAX_VIEWS) return fail(GEOCACHE_ESHAPE, "N=%d out of range [1, %d]", N, GEOCACHE_MAX_VIEWS);
+    if (a < 1 || a > N) return fail(GEOCACHE_EINVAL, "a=%d must be in [1, N=%d]", a, N);
+    int full = geocache_is_full_step(step, S, sched);
+    if (full < 0) return full;
+    int ordinal = 0;
+    for (int t = 0; t < step; ++t) {
+        const int f = geocache_is_full_step(t, S, sched);
+        if (f < 0) return f;
+        ordinal += f ? 0 : 1;
+    }
+    int cand[GEOCACHE_MAX_VIEWS];
+    if (sched->contiguous_rotation) {
+        for (int j = 0; j < a; ++j) cand[j] = (int)(((long long)ordinal * a + j) % N);
+    } else {
+        const int s = (N + a - 1) / a;
+        const int r = ordinal % s;
+        for (int j = 0; j < a; ++j) cand[j] = (r + j * s) % N;
+    }
+    bool used[GEOCACHE_MAX_VIEWS] = {false};
+    bool in_cand[GEOCACHE_MAX_VIEWS] = {false};
+    for (int j = 0; j < a; ++j) in_cand[cand[j]] = true;
+    int out[GEOCACHE_MAX_VIEWS];
+    for (int j = 0; j < a; ++j) {
+        int x = cand[j];
+        if (used[x]) {
+            x = -1;
+            for (int y = 0; y < N; ++y)
+                if (!used[y] && !in_cand[y]) { x = y; break; }
+            if (x < 0)
+                for (int y = 0; y < N; ++y)
+                    if (!used[y]) { x = y; break; }
+        }
+        used[x] = true;
+        out[j] = x;
+    }
+    // ascending order
+    for (int i = 1; i < a; ++i)
+        for (int j = i; j > 0 && out[j - 1] > out[j]; --j) { int tmp = out[j]; out[j] = out[j - 1]; out[j - 1] = tmp; }
+    for (int j = 0; j < a; ++j) anchors_out[j] = out[j];
+    if (is_full_out) *is_full_out = full;
+    return ok();
+}
+
+}  // extern "C"

@@ -1,0 +1,113 @@
+// Device-side geometry of the correspondence operator G_{u->v} (Sec. 3.2,
+// "Correspondence operator"): projection of a target token's 3-D position
+// into a source camera, choice of the K taps, the per-tap tolerance test and
+// the renormalised area weights.
+//
+// The same functions serve the table build and the on-the-fly taps of the
+// transport kernel, so both produce identical indices and weights.  Every
+// operation that feeds an integer decision (projection, floor, tolerance
+// test) is an explicitly rounded binary32 intrinsic in a fixed order, so no
+// multiply-add is ever contracted and the decisions do not depend on how the
+// compiler schedules the code.
+#pragma once
+
+#include <cstdint>
+
+#include "geocache.h"
+
+namespace geocache {
+
+struct Taps {
+    int32_t q[4];   // source token index row*W + col, -1 = not kept
+    float w[4];     // renormalised weight, 0 where not kept
+    int kept;       // number of kept taps
+};
+
+__device__ __forceinline__ void taps_clear(Taps& t) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) { t.q[k] = -1; t.w[k] = 0.0f; }
+    t.kept = 0;
+}
+
+// x_c = R X + t with each row summed ((R0 X0 + R1 X1) + R2 X2) + t, then the
+// pinhole projection.  Returns false when the point is not in front.
+__device__ __forceinline__ bool project(const geocache_camera& c, float X0, float X1, float X2,
+                                        float& uu, float& vv) {
+    float xc[3];
+#pragma unroll
+    for (int r = 0; r < 3; ++r) {
+        float s = __fmul_rn(c.R[3 * r], X0);
+        s = __fadd_rn(s, __fmul_rn(c.R[3 * r + 1], X1));
+        s = __fadd_rn(s, __fmul_rn(c.R[3 * r + 2], X2));
+        xc[r] = __fadd_rn(s, c.t[r]);
+    }
+    if (!(xc[2] > 0.0f)) return false;
+    uu = __fadd_rn(__fmul_rn(c.fx, __fdiv_rn(xc[0], xc[2])), c.cx);
+    vv = __fadd_rn(__fmul_rn(c.fy, __fdiv_rn(xc[1], xc[2])), c.cy);
+    return true;
+}
+
+__device__ __forceinline__ float sqdist(const float* P, float X0, float X1, float X2) {
+    const float dx = __fsub_rn(__ldg(P + 0), X0);
+    const float dy = __fsub_rn(__ldg(P + 1), X1);
+    const float dz = __fsub_rn(__ldg(P + 2), X2);
+    return __fadd_rn(__fadd_rn(__fmul_rn(dx, dx), __fmul_rn(dy, dy)), __fmul_rn(dz, dz));
+}
+
+// Taps of target point X in source view u (pos_u [H*W*3], valid_u [H*W]).
+// K = 4: the bilinear footprint TL, TR, BL, BR around the projection with
+// weights (1-fx)(1-fy), fx(1-fy), (1-fx)fy, fx fy; K = 1: the token
+// containing the projection with weight 1.  A tap is kept iff it is inside
+// the image, its texel is foreground, its weight factors are non-zero and
+// ||P_u(q) - X||^2 <= tau2.  Kept weights are divided by their sum.
+template <int K>
+__device__ __forceinline__ void compute_taps(const geocache_camera& cam, const float* __restrict__ pos_u,
+                                             const uint8_t* __restrict__ valid_u, int H, int W,
+                                             float X0, float X1, float X2, float tau2, Taps& t) {
+    taps_clear(t);
+    float uu, vv;
+    if (!project(cam, X0, X1, X2, uu, vv)) return;
+    if (K == 1) {
+        if (!(uu >= 0.0f && uu < (float)W && vv >= 0.0f && vv < (float)H)) return;
+        const int col = (int)floorf(uu), row = (int)floorf(vv);
+        const int q = row * W + col;
+        if (!__ldg(valid_u + q)) return;
+        if (!(sqdist(pos_u + 3 * (size_t)q, X0, X1, X2) <= tau2)) return;
+        t.q[0] = q;
+        t.w[0] = 1.0f;
+        t.kept = 1;
+        return;
+    } else {
+        const float x = __fsub_rn(uu, 0.5f), y = __fsub_rn(vv, 0.5f);
+        if (!(x >= -1.0f && x < (float)W && y >= -1.0f && y < (float)H)) return;
+        const float i0f = floorf(x), j0f = floorf(y);
+        const int i0 = (int)i0f, j0 = (int)j0f;
+        const float fx = __fsub_rn(x, i0f), fy = __fsub_rn(y, j0f);
+        const float ax[2] = {__fsub_rn(1.0f, fx), fx};
+        const float ay[2] = {__fsub_rn(1.0f, fy), fy};
+        float raw[4];
+        float sum = 0.0f;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const int di = k & 1, dj = k >> 1;
+            const int col = i0 + di, row = j0 + dj;
+            raw[k] = 0.0f;
+            if (col < 0 || col >= W || row < 0 || row >= H) continue;
+            if (ax[di] == 0.0f || ay[dj] == 0.0f) continue;
+            const int q = row * W + col;
+            if (!__ldg(valid_u + q)) continue;
+            if (!(sqdist(pos_u + 3 * (size_t)q, X0, X1, X2) <= tau2)) continue;
+            raw[k] = __fmul_rn(ax[di], ay[dj]);
+            t.q[k] = q;
+            sum = __fadd_rn(sum, raw[k]);
+            ++t.kept;
+        }
+        if (t.kept) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+                if (t.q[k] >= 0) t.w[k] = __fdiv_rn(raw[k], sum);
+        }
+    }
+}
+
+}  // namespace geocache

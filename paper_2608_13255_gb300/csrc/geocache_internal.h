@@ -1,0 +1,53 @@
+// Internal interface between the C ABI layer (geocache_api.cu) and the
+// kernels (geocache_kernels.cu).  Not installed; not part of the ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "geocache.h"
+
+namespace geocache {
+
+// Per-step sampler constants, formed in double on the host and rounded once.
+struct ReconCoef {
+    int enabled;     // 0: transport only
+    int sampler;     // GEOCACHE_DDIM / GEOCACHE_FM_EULER
+    int pred_kind;   // geocache_pred
+    float st, s1t, inv_s1t, sp, s1p;   // DDIM: sqrt(ab_t), sqrt(1-ab_t), 1/sqrt(1-ab_t), sqrt(ab_prev), sqrt(1-ab_prev)
+    float inv_sigma, dsigma;           // FM: 1/sigma, sigma_next - sigma
+};
+
+struct TransportArgs {
+    int B, N, H, W, C, K, a;
+    int c0, cn;                         // channel window [c0, c0 + cn) handled by this launch
+    int mode;                           // geocache_corr_mode
+    int write_anchor_rows;              // 0 when x0_out aliases x0_prev (rows written afterwards)
+    int lat_dtype;                      // geocache_dtype
+    const float* pos;
+    const uint8_t* valid;
+    const geocache_camera* cams;
+    const float* tau;
+    const int32_t* idx;
+    const float* w;
+    const float* x0_new;
+    const float* x0_prev;
+    float* x0_out;
+    const void* x_t;
+    void* x_next;
+    float* pred_out;
+    ReconCoef coef;
+    int32_t anchors[GEOCACHE_MAX_VIEWS];
+    int32_t slot_of[GEOCACHE_MAX_VIEWS];   // slot in `anchors`, -1 for non-anchors
+};
+
+cudaError_t launch_tau(const float* pos, const uint8_t* valid, int B, int N, int H, int W,
+                       float tol_frac, float* tau, cudaStream_t s);
+cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s);
+cudaError_t launch_transport(const TransportArgs& t, cudaStream_t s);
+cudaError_t launch_copy_anchor_rows(const TransportArgs& t, cudaStream_t s);
+cudaError_t launch_reconstruct(const void* x_t, const float* x0, void* x_next, int lat_dtype, int64_t n,
+                               const ReconCoef& coef, float* pred_out, float* x0_store, cudaStream_t s);
+
+}  // namespace geocache

@@ -1,0 +1,262 @@
+"""ctypes binding of libgeocache.so (include/geocache.h).
+
+Same entry points as the C ABI; this module only marshals arguments (torch
+tensors -> device pointers, dicts -> C structs, the current torch stream) and
+checks that tensor shapes, dtypes and devices match what the C call will
+read and write, since the C layer only sees pointers.  All computation runs
+in the library's CUDA kernels; there is no fallback: if the library has not
+been built, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+OK, EINVAL, ESHAPE, EDTYPE, ECUDA, ETIMEOUT, EDEVICE, EALIAS = 0, -1, -2, -3, -4, -5, -6, -7
+F32, BF16 = 0, 1
+DDIM, FM_EULER = 0, 1
+PRED_NONE, PRED_EPS, PRED_V, PRED_VELOCITY = 0, 1, 2, 3
+CORR_GEOMETRY, CORR_TABLE = 0, 1
+SCHED_EVERY_K, SCHED_HEAD_MID_TAIL, SCHED_LIST, SCHED_ALL_FULL, SCHED_SINGLE_CACHED = 0, 1, 2, 3, 4
+MAX_VIEWS = 64
+
+_SAMPLERS = {"ddim": DDIM, "fm_euler": FM_EULER, DDIM: DDIM, FM_EULER: FM_EULER}
+_PREDS = {None: PRED_NONE, "none": PRED_NONE, "eps": PRED_EPS, "v": PRED_V, "velocity": PRED_VELOCITY,
+          PRED_NONE: PRED_NONE, PRED_EPS: PRED_EPS, PRED_V: PRED_V, PRED_VELOCITY: PRED_VELOCITY}
+
+
+class GeocacheError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__("geocache status %d: %s" % (status, msg))
+        self.status = status
+
+
+class Camera(ctypes.Structure):
+    _fields_ = [("R", ctypes.c_float * 9), ("t", ctypes.c_float * 3), ("fx", ctypes.c_float),
+                ("fy", ctypes.c_float), ("cx", ctypes.c_float), ("cy", ctypes.c_float)]
+
+
+class Corr(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int), ("N", ctypes.c_int), ("H", ctypes.c_int), ("W", ctypes.c_int),
+                ("K", ctypes.c_int), ("tol_frac", ctypes.c_float),
+                ("pos", ctypes.c_void_p), ("valid", ctypes.c_void_p), ("cams", ctypes.c_void_p),
+                ("tau", ctypes.c_void_p), ("idx", ctypes.c_void_p), ("w", ctypes.c_void_p),
+                ("mode", ctypes.c_int)]
+
+
+class Recon(ctypes.Structure):
+    _fields_ = [("sampler", ctypes.c_int), ("a_t", ctypes.c_double), ("a_prev", ctypes.c_double),
+                ("sigma", ctypes.c_double), ("sigma_next", ctypes.c_double), ("pred_kind", ctypes.c_int),
+                ("pred_out", ctypes.c_void_p)]
+
+
+class Schedule(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int), ("k", ctypes.c_int), ("head", ctypes.c_int), ("mid", ctypes.c_int),
+                ("tail", ctypes.c_int), ("full_steps", ctypes.c_void_p), ("n_full_steps", ctypes.c_int),
+                ("contiguous_rotation", ctypes.c_int)]
+
+
+assert ctypes.sizeof(Camera) == 64
+
+_LIB = None
+EXPORTS = ("geocache_build_corr", "geocache_transport_step", "geocache_reconstruct", "geocache_is_full_step",
+           "geocache_rotate_anchors", "geocache_last_error", "geocache_abi_version")
+
+
+def lib_path() -> str:
+    return _build.LIB
+
+
+def load():
+    """Load libgeocache.so; raise if it has not been built."""
+    global _LIB
+    if _LIB is None:
+        path = lib_path()
+        if not os.path.exists(path):
+            raise RuntimeError("libgeocache.so is not built (%s); run __graft_entry__.build() or "
+                               "python -m paper_2608_13255_gb300.build" % path)
+        L = ctypes.CDLL(path)
+        P, i, i64 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64
+        L.geocache_build_corr.argtypes = [ctypes.POINTER(Corr), P]
+        L.geocache_transport_step.argtypes = [ctypes.POINTER(Corr), P, i, i, P, P, P, P, P, i,
+                                              ctypes.POINTER(Recon), P]
+        L.geocache_reconstruct.argtypes = [P, P, P, i, i64, ctypes.POINTER(Recon), P, P]
+        L.geocache_is_full_step.argtypes = [i, i, ctypes.POINTER(Schedule)]
+        L.geocache_rotate_anchors.argtypes = [i, i, i, i, ctypes.POINTER(Schedule), P, ctypes.POINTER(i)]
+        L.geocache_last_error.restype = ctypes.c_char_p
+        L.geocache_last_error.argtypes = []
+        L.geocache_abi_version.argtypes = []
+        for name in EXPORTS[:5]:
+            getattr(L, name).restype = ctypes.c_int
+        L.geocache_abi_version.restype = ctypes.c_int
+        _LIB = L
+    return _LIB
+
+
+def last_error() -> str:
+    return load().geocache_last_error().decode()
+
+
+def _check(status: int):
+    if status != OK:
+        raise GeocacheError(status, last_error())
+    return status
+
+
+def _stream(stream):
+    if stream is None:
+        return ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def _dev(t, dtype, numel=None, name="tensor"):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("%s must be a torch tensor" % name)
+    if not t.is_cuda:
+        raise ValueError("%s must be on a CUDA device" % name)
+    if t.dtype != dtype:
+        raise TypeError("%s must be %s (got %s)" % (name, dtype, t.dtype))
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    if numel is not None and t.numel() != numel:
+        raise ValueError("%s has %d elements, expected %d" % (name, t.numel(), numel))
+    return t.data_ptr()
+
+
+def _lat_dtype(t):
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise TypeError("latents must be float32 or bfloat16 (got %s)" % t.dtype)
+
+
+# ------------------------------------------------------------- structs --
+class CorrHandle:
+    """A filled geocache_corr plus references to the tensors it points to."""
+
+    def __init__(self, c: Corr, keep):
+        self.c = c
+        self._keep = keep
+
+    @property
+    def tau(self):
+        return self._keep["tau"]
+
+    @property
+    def idx(self):
+        return self._keep.get("idx")
+
+    @property
+    def w(self):
+        return self._keep.get("w")
+
+
+def make_corr(pos, valid, cams, tau, idx=None, w=None, K=4, tol_frac=0.01, mode=None) -> CorrHandle:
+    """Describe a batch's geometry (and optional tables) for the C ABI."""
+    B, N, H, W = valid.shape
+    n = B * N * H * W
+    keep = {"pos": pos, "valid": valid, "cams": cams, "tau": tau, "idx": idx, "w": w}
+    c = Corr(B, N, H, W, K, tol_frac,
+             _dev(pos, torch.float32, 3 * n, "pos"), _dev(valid, torch.uint8, n, "valid"),
+             _dev(cams, torch.float32, 16 * B * N, "cams"), _dev(tau, torch.float32, B, "tau"),
+             _dev(idx, torch.int32, n * N * K, "idx"), _dev(w, torch.float32, n * N * K, "w"),
+             (CORR_TABLE if idx is not None else CORR_GEOMETRY) if mode is None else mode)
+    return CorrHandle(c, keep)
+
+
+def make_recon(sampler="ddim", a_t=0.0, a_prev=0.0, sigma=0.0, sigma_next=0.0, pred_kind=None,
+               pred_out=None) -> Recon:
+    r = Recon(_SAMPLERS[sampler], float(a_t), float(a_prev), float(sigma), float(sigma_next),
+              _PREDS[pred_kind], None if pred_out is None else _dev(pred_out, torch.float32, name="pred_out"))
+    r._pred = pred_out  # keeps the tensor alive; its size is checked at the call
+    return r
+
+
+def _check_pred(recon, n):
+    t = getattr(recon, "_pred", None) if recon is not None else None
+    if t is not None and t.numel() != n:
+        raise ValueError("pred_out has %d elements, expected %d" % (t.numel(), n))
+
+
+_SCHED_KINDS = {"every_k": SCHED_EVERY_K, "head_mid_tail": SCHED_HEAD_MID_TAIL, "list": SCHED_LIST,
+                "all_full": SCHED_ALL_FULL, "single_cached": SCHED_SINGLE_CACHED}
+
+
+def make_schedule(spec: dict):
+    kind = _SCHED_KINDS[spec["kind"]]
+    steps = (ctypes.c_int32 * max(1, len(spec.get("steps", ()))))(*spec.get("steps", ()))
+    s = Schedule(kind, int(spec.get("k", 1)), int(spec.get("head", 2)), int(spec.get("mid", 1)),
+                 int(spec.get("tail", 1)), ctypes.cast(steps, ctypes.c_void_p), len(spec.get("steps", ())),
+                 int(spec.get("contiguous", 0)))
+    return s, steps
+
+
+# ---------------------------------------------------------- entry points --
+def build_corr(corr: CorrHandle, stream=None) -> CorrHandle:
+    """geocache_build_corr: tau (and the tables if the handle has idx/w)."""
+    _check(load().geocache_build_corr(ctypes.byref(corr.c), _stream(stream)))
+    return corr
+
+
+def transport_step(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev, x0_out, x_t=None, x_next=None,
+                   recon: Recon | None = None, stream=None):
+    """geocache_transport_step on torch tensors (see include/geocache.h)."""
+    c = corr.c
+    anc = sorted(int(a) for a in anchors)
+    a = len(anc)
+    n_all = c.B * c.N * C * c.H * c.W
+    arr = (ctypes.c_int32 * max(1, a))(*anc)
+    lat = F32
+    pt = pn = None
+    if recon is not None:
+        lat = _lat_dtype(x_t)
+        dt = x_t.dtype
+        pt, pn = _dev(x_t, dt, n_all, "x_t"), _dev(x_next, dt, n_all, "x_next")
+        _check_pred(recon, n_all)
+    st = load().geocache_transport_step(
+        ctypes.byref(c), ctypes.cast(arr, ctypes.c_void_p), a, int(C),
+        _dev(x0_anchor_new, torch.float32, c.B * a * C * c.H * c.W, "x0_anchor_new"),
+        _dev(x0_prev, torch.float32, n_all, "x0_prev"), _dev(x0_out, torch.float32, n_all, "x0_out"),
+        pt, pn, lat, ctypes.byref(recon) if recon is not None else None, _stream(stream))
+    _check(st)
+
+
+def reconstruct(x_t, x0, x_next, recon: Recon, x0_store=None, stream=None):
+    """geocache_reconstruct (full-step passthrough) on torch tensors."""
+    n = x0.numel()
+    dt = x_t.dtype
+    _check_pred(recon, n)
+    _check(load().geocache_reconstruct(_dev(x_t, dt, n, "x_t"), _dev(x0, torch.float32, n, "x0"),
+                                       _dev(x_next, dt, n, "x_next"), _lat_dtype(x_t), n, ctypes.byref(recon),
+                                       _dev(x0_store, torch.float32, n, "x0_store"), _stream(stream)))
+
+
+def is_full_step(step: int, S: int, sched: dict) -> bool:
+    s, _keep = make_schedule(sched)
+    r = load().geocache_is_full_step(int(step), int(S), ctypes.byref(s))
+    if r < 0:
+        raise GeocacheError(r, last_error())
+    return bool(r)
+
+
+def rotate_anchors(N: int, a: int, step: int, S: int, sched: dict):
+    """(anchors, is_full) of a step."""
+    s, _keep = make_schedule(sched)
+    out = (ctypes.c_int32 * a)()
+    full = ctypes.c_int(0)
+    _check(load().geocache_rotate_anchors(int(N), int(a), int(step), int(S), ctypes.byref(s),
+                                          ctypes.cast(out, ctypes.c_void_p), ctypes.byref(full)))
+    return list(out), bool(full.value)
+
+
+def abi_version() -> int:
+    return load().geocache_abi_version()

@@ -1,0 +1,121 @@
+"""Shared plumbing of the GPU tests: seeded step inputs, device uploads and
+the parity tolerances.
+
+Tolerances (from the required bar: latents within 1e-5 relative in fp32 and
+2e-2 absolute in bf16; indices bit-exact):
+* fp32 values (x0 cache, fp32 latents, weights): |gpu - ref| <= 1e-5 * max(|ref|, 1).
+  The floor at unit scale is needed because latents are unit-variance and a
+  transported sum can cancel to ~0, where a purely relative bound is
+  meaningless; the kernels' float arithmetic errs by a few ulp of the
+  operands (<1e-6 at unit scale).
+* bf16 latents: |gpu - ref| <= 2e-2 against the oracle's unrounded binary64
+  value, and at most one bf16 ulp away from the oracle's own rounding (the
+  kernel rounds a float result, the oracle a binary64 one, so a tie can land
+  one ulp apart).
+* predictions (eps, v): the conversion divides by sqrt(1 - ab_t), which
+  magnifies the error of x0 by sqrt(ab_t)/sqrt(1 - ab_t); the bound is
+  1e-5 * (1 + sqrt(ab_t)/sqrt(1 - ab_t)) * max(|ref|, 1).
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2608_13255_gb300 import synth
+
+RTOL = 1e-5
+BF16_ATOL = 2e-2
+
+
+def assert_f32_close(got, ref, scale=1.0, what=""):
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    err = np.abs(got - ref)
+    bound = RTOL * scale * np.maximum(np.abs(ref), 1.0)
+    bad = err > bound
+    assert not bad.any(), "%s: %d/%d outside tolerance, worst %.3g at %s (got %r, ref %r)" % (
+        what, bad.sum(), bad.size, err.max(), np.unravel_index(err.argmax(), err.shape),
+        got.reshape(-1)[err.argmax()], ref.reshape(-1)[err.argmax()])
+    return float(err.max())
+
+
+def bf16_to_f64(bits):
+    return (np.asarray(bits, np.uint16).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def _ordered(bits):
+    b = np.asarray(bits, np.uint16).astype(np.int32)
+    return np.where(b & 0x8000, 0x8000 - b, b)  # monotone integer order of bf16 values
+
+
+def assert_bf16_close(got_bits, ref64, what=""):
+    got = bf16_to_f64(got_bits)
+    err = np.abs(got - ref64)
+    assert err.max() <= BF16_ATOL, "%s: max |err| %.4g > %.3g" % (what, err.max(), BF16_ATOL)
+    ulps = np.abs(_ordered(got_bits) - _ordered(oracle.round_bf16(ref64)))
+    assert ulps.max() <= 1, "%s: %d elements more than one bf16 ulp from the oracle" % (what, (ulps > 1).sum())
+    return float(err.max()), float((ulps == 1).mean())
+
+
+def lat_torch_dtype(w):
+    return torch.bfloat16 if w.dtype == "bf16" else torch.float32
+
+
+def latent_values(x32, w):
+    """Latent array as the GPU stores it (bf16-rounded for bf16 workloads),
+    returned as float64 values for the oracle and as a torch tensor."""
+    if w.dtype == "bf16":
+        bits = synth.to_bf16_bits(x32)
+        t = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16)
+        return bf16_to_f64(bits), t
+    return x32.astype(np.float64), torch.from_numpy(np.ascontiguousarray(x32))
+
+
+def step_inputs(w, step, anchors, seed_extra=0):
+    """x0_prev [B,N,C,H,W] f32, x0_new [B,a,C,H,W] f32 and x_t (float32 before
+    storage rounding) for one step of a workload."""
+    rng = np.random.default_rng(np.random.SeedSequence([w.seed, 77, step, seed_extra]))
+    shp = (w.B, w.N, w.C, w.H, w.W)
+    x0_prev = rng.standard_normal(shp, dtype=np.float32)
+    x0_new = x0_prev[:, anchors] + synth.delta(w, step, anchors)
+    x_t = rng.standard_normal(shp, dtype=np.float32)
+    return x0_prev, np.ascontiguousarray(x0_new, dtype=np.float32), x_t
+
+
+def recon_kw(params, pred=None):
+    """Arguments for the oracle's reconstruction from a synth.recon_params dict."""
+    r = dict(sampler=oracle.DDIM if params["sampler"] == "ddim" else oracle.FM_EULER,
+             a_t=params.get("a_t", 0.0), a_prev=params.get("a_prev", 0.0),
+             sigma=params.get("sigma", 0.0), sigma_next=params.get("sigma_next", 0.0),
+             pred_kind={None: 0, "eps": 1, "v": 2, "velocity": 3}[pred])
+    return r
+
+
+def pred_scale(params):
+    if params["sampler"] == "ddim":
+        a = params["a_t"]
+        return 1.0 + math.sqrt(a) / math.sqrt(1.0 - a)
+    return 1.0 + 1.0 / params["sigma"]
+
+
+class DeviceGeometry:
+    """A workload's geometry on the GPU, with tau and (optionally) tables."""
+
+    def __init__(self, w, K=4, tables=True, dev="cuda"):
+        from paper_2608_13255_gb300 import geocache as gc
+        self.w = w
+        self.pos = torch.from_numpy(w.pos).to(dev)
+        self.valid = torch.from_numpy(w.valid).to(dev)
+        self.cams = torch.from_numpy(w.cams).to(dev)
+        self.tau = torch.zeros(w.B, dtype=torch.float32, device=dev)
+        self.idx = self.wt = None
+        if tables:
+            shp = (w.B, w.N, w.N, w.H, w.W, K)
+            self.idx = torch.empty(shp, dtype=torch.int32, device=dev)
+            self.wt = torch.empty(shp, dtype=torch.float32, device=dev)
+        self.corr = gc.make_corr(self.pos, self.valid, self.cams, self.tau, self.idx, self.wt, K=K,
+                                 tol_frac=w.tol_frac, mode=gc.CORR_GEOMETRY)
+        gc.build_corr(self.corr)
