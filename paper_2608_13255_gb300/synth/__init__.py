@@ -384,7 +384,7 @@ def make_workload(name: str, **overrides) -> Workload:
     views = _layout(w.layout, w.N)
     assert len(views) == w.N, (name, len(views), w.N)
     cams1 = np.stack([look_at_camera(az, el, w.H, w.W) for az, el in views], 0)
-    w.cams = np.array(np.broadcast_to(cams1, (w.B, w.N, CAM_FLOATS)), dtype=np.float32, copy=True)
+    w.cams = np.ascontiguousarray(np.tile(cams1[None], (w.B, 1, 1)), dtype=np.float32)
     w.pos = np.zeros((w.B, w.N, w.H, w.W, 3), np.float32)
     w.valid = np.zeros((w.B, w.N, w.H, w.W), np.uint8)
     cache = {}
