@@ -42,7 +42,7 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="batch128")
     p.add_argument("--assets", type=int, default=64, help="assets per GPU (the batch128 sweep axis)")
-    p.add_argument("--corr", default="geometry", choices=["geometry", "table"])
+    p.add_argument("--corr", default="mask", choices=["mask", "geometry", "table"])
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-assets", type=int, default=4, help="assets in the oracle's timed sample")
@@ -84,7 +84,7 @@ def step_bytes(w):
 class Trajectory:
     """Device state of one batch's trajectory and the loop over its steps."""
 
-    def __init__(self, w, dev, corr_mode="geometry"):
+    def __init__(self, w, dev, corr_mode="mask"):
         import torch
         from paper_2608_13255_gb300 import geocache as gc
         from paper_2608_13255_gb300 import synth
@@ -94,13 +94,16 @@ class Trajectory:
         self.valid = torch.from_numpy(w.valid).to(dev)
         self.cams = torch.from_numpy(w.cams).to(dev)
         self.tau = torch.zeros(w.B, dtype=torch.float32, device=dev)
-        idx = wt = None
+        idx = wt = keep = None
         if corr_mode == "table":
             shp = (w.B, w.N, w.N, w.H, w.W, w.K)
             idx = torch.empty(shp, dtype=torch.int32, device=dev)
             wt = torch.empty(shp, dtype=torch.float32, device=dev)
+        if corr_mode == "mask":
+            keep = torch.empty((w.B, w.N, w.N, w.H, w.W), dtype=torch.uint8, device=dev)
+        mode = {"mask": gc.CORR_MASK, "table": gc.CORR_TABLE, "geometry": gc.CORR_GEOMETRY}[corr_mode]
         self.corr = gc.make_corr(self.pos, self.valid, self.cams, self.tau, idx, wt, K=w.K, tol_frac=w.tol_frac,
-                                 mode=gc.CORR_TABLE if corr_mode == "table" else gc.CORR_GEOMETRY)
+                                 mode=mode, keep=keep)
         xT, x0 = synth.initial_latents(w)
         lat = torch.bfloat16 if w.dtype == "bf16" else torch.float32
         self.x = torch.from_numpy(xT).to(dev).to(lat)
@@ -136,7 +139,7 @@ class Trajectory:
         gc, w = self.gc, self.w
         launches = 0
         gc.build_corr(self.corr)
-        launches += 1 + (1 if self.corr.idx is not None else 0)
+        launches += 1 + (1 if (self.corr.idx is not None or self.corr.keep is not None) else 0)
         cache = None
         for t in range(w.S):
             anchors, full = gc.rotate_anchors(w.N, w.a, t, w.S, self.sched)
@@ -154,7 +157,7 @@ class Trajectory:
                 if events is not None:
                     e1.record()
                     events.append((e0, e1))
-                launches += (w.C + 15) // 16 if w.C > 4 else 1
+                launches += gc.transport_launches(w.a, w.C, in_place=False)
                 cache = out
         return launches
 

@@ -55,10 +55,13 @@ typedef enum {
     GEOCACHE_PRED_VELOCITY = 3  /* FM: u = (x_sigma - x0) / sigma */
 } geocache_pred;
 
-/* How geocache_transport_step obtains the taps of G_{u->v}. */
+/* How geocache_transport_step obtains the taps of G_{u->v}.  All three give
+ * bit-identical taps and weights. */
 typedef enum {
-    GEOCACHE_CORR_GEOMETRY = 0, /* recompute them from pos/valid/cams/tau (bit-identical to the tables) */
-    GEOCACHE_CORR_TABLE = 1     /* read idx/w written by geocache_build_corr (or supplied by the caller) */
+    GEOCACHE_CORR_GEOMETRY = 0, /* recompute every tap test from pos/valid/cams/tau */
+    GEOCACHE_CORR_TABLE = 1,    /* read idx/w written by geocache_build_corr (or supplied by the caller) */
+    GEOCACHE_CORR_MASK = 2      /* read the 1-byte keep masks written by geocache_build_corr; recompute
+                                   the projection and weights only where a tap is kept (fastest) */
 } geocache_corr_mode;
 
 /* Pinhole camera, world -> camera: x_c = R x_w + t (R row-major), +z forward,
@@ -90,6 +93,7 @@ typedef struct {
     int32_t* idx;                   /* device [B,N(v),N(u),H,W,K] i32 source token index row*W+col,
                                        -1 = tap not kept; or NULL (tables not built) */
     float* w;                       /* device [B,N(v),N(u),H,W,K] f32 weights, 0 where idx = -1; or NULL */
+    uint8_t* keep;                  /* device [B,N(v),N(u),H,W] u8: bit k set iff tap k is kept; or NULL */
     geocache_corr_mode mode;        /* taps used by geocache_transport_step */
 } geocache_corr;
 
@@ -133,9 +137,10 @@ typedef struct {
  * geocache_build_corr -- tau and the correspondence tables (Sec. 3.2,
  * "Correspondence operator"; precomputed once per asset).
  *
- * Reads corr->pos, corr->valid, corr->cams; writes corr->tau[B] and, when
- * corr->idx and corr->w are both non-NULL, the tables for every ordered pair
- * (v, u): the diagonal u == v and background targets hold idx -1 / w 0.
+ * Reads corr->pos, corr->valid, corr->cams; writes corr->tau[B] and, for
+ * every ordered pair (v, u), the tables idx/w (when both are non-NULL) and
+ * the keep masks (when keep is non-NULL): the diagonal u == v and
+ * background targets hold idx -1 / w 0 / keep 0.
  * Sizes: 1 <= B, 2 <= N <= GEOCACHE_MAX_VIEWS, 1 <= H, W <= 16384,
  * K in {1, 4}, 0 < tol_frac.  tau must not overlap the other buffers.
  * Returns GEOCACHE_OK, EINVAL (NULL / bad K / tol_frac), ESHAPE, ECUDA.
@@ -165,8 +170,8 @@ int geocache_build_corr(geocache_corr* corr, void* stream);
  *             view (bf16 stores round to nearest even); x_next may equal x_t.
  *             Ignored when recon is NULL.
  *   C         1 <= C <= GEOCACHE_MAX_CHANNELS.
- * corr must have been filled by geocache_build_corr (tau, and idx/w in
- * GEOCACHE_CORR_TABLE mode).
+ * corr must have been filled by geocache_build_corr (tau; idx/w in
+ * GEOCACHE_CORR_TABLE mode; keep in GEOCACHE_CORR_MASK mode).
  * Returns GEOCACHE_OK, EINVAL, ESHAPE, EDTYPE, EALIAS, ECUDA.
  * ------------------------------------------------------------------------ */
 int geocache_transport_step(const geocache_corr* corr, const int32_t* anchors, int a, int C,

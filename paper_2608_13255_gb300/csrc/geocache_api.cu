@@ -114,11 +114,16 @@ int geocache_build_corr(geocache_corr* c, void* stream) {
         if (c->K == 4 && (((uintptr_t)c->idx | (uintptr_t)c->w) & 15))
             return fail(GEOCACHE_EINVAL, "idx and w must be 16-byte aligned for K=4");
         if (overlap(c->idx, rows * 4, c->w, rows * 4)) return fail(GEOCACHE_EALIAS, "idx and w overlap");
+        if (c->keep && (overlap(c->keep, rows / c->K, c->idx, rows * 4) || overlap(c->keep, rows / c->K, c->w, rows * 4)))
+            return fail(GEOCACHE_EALIAS, "keep overlaps idx or w");
     }
+    if (c->keep && (overlap(c->keep, texels * c->N, c->pos, texels * 12) || overlap(c->keep, texels * c->N, c->valid, texels) ||
+                    overlap(c->keep, texels * c->N, c->tau, sizeof(float) * c->B)))
+        return fail(GEOCACHE_EALIAS, "keep overlaps an input");
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = geocache::launch_tau(c->pos, c->valid, c->B, c->N, c->H, c->W, c->tol_frac, c->tau, s);
     if (e != cudaSuccess) return cuda_fail(e, "tau kernel launch");
-    if (c->idx) {
+    if (c->idx || c->keep) {
         e = geocache::launch_build_corr(*c, s);
         if (e != cudaSuccess) return cuda_fail(e, "correspondence kernel launch");
     }
@@ -138,6 +143,9 @@ int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int 
             return fail(GEOCACHE_EINVAL, "geometry mode needs pos, valid, cams and tau");
     } else if (c->mode == GEOCACHE_CORR_TABLE) {
         if (!c->idx || !c->w) return fail(GEOCACHE_EINVAL, "table mode needs idx and w");
+    } else if (c->mode == GEOCACHE_CORR_MASK) {
+        if (!c->keep || !c->pos || !c->valid || !c->cams || !c->tau)
+            return fail(GEOCACHE_EINVAL, "mask mode needs keep, pos, valid, cams and tau");
     } else {
         return fail(GEOCACHE_EINVAL, "unknown corr mode %d", (int)c->mode);
     }
@@ -177,23 +185,19 @@ int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int 
     t.write_anchor_rows = (x0_out != x0_prev);
     t.lat_dtype = lat_dtype;
     t.pos = c->pos; t.valid = c->valid; t.cams = c->cams; t.tau = c->tau; t.idx = c->idx; t.w = c->w;
+    t.keep = c->keep;
     t.x0_new = x0_anchor_new; t.x0_prev = x0_prev; t.x0_out = x0_out;
     t.x_t = x_t; t.x_next = x_next; t.pred_out = recon ? recon->pred_out : nullptr;
     t.coef = coef;
     for (int v = 0; v < GEOCACHE_MAX_VIEWS; ++v) { t.slot_of[v] = -1; t.anchors[v] = -1; }
     for (int s = 0; s < a; ++s) { t.anchors[s] = anchors[s]; t.slot_of[anchors[s]] = s; }
     cudaStream_t s = (cudaStream_t)stream;
-    const int chunk = C <= 4 ? 4 : 16;
-    for (int c0 = 0; c0 < C; c0 += chunk) {
-        t.c0 = c0;
-        t.cn = C - c0 < chunk ? C - c0 : chunk;
-        cudaError_t e = geocache::launch_transport(t, s);
-        if (e != cudaSuccess) return cuda_fail(e, "transport kernel launch");
-    }
+    t.c0 = 0;
+    t.cn = C;
+    cudaError_t e = geocache::launch_transport(t, s);
+    if (e != cudaSuccess) return cuda_fail(e, "transport kernel launch");
     if (!t.write_anchor_rows) {
-        t.c0 = 0;
-        t.cn = C;
-        cudaError_t e = geocache::launch_copy_anchor_rows(t, s);
+        e = geocache::launch_copy_anchor_rows(t, s);
         if (e != cudaSuccess) return cuda_fail(e, "anchor-row copy launch");
     }
     return ok();

@@ -54,60 +54,104 @@ __device__ __forceinline__ float sqdist(const float* P, float X0, float X1, floa
     return __fadd_rn(__fadd_rn(__fmul_rn(dx, dx), __fmul_rn(dy, dy)), __fmul_rn(dz, dz));
 }
 
-// Taps of target point X in source view u (pos_u [H*W*3], valid_u [H*W]).
-// K = 4: the bilinear footprint TL, TR, BL, BR around the projection with
-// weights (1-fx)(1-fy), fx(1-fy), (1-fx)fy, fx fy; K = 1: the token
-// containing the projection with weight 1.  A tap is kept iff it is inside
-// the image, its texel is foreground, its weight factors are non-zero and
-// ||P_u(q) - X||^2 <= tau2.  Kept weights are divided by their sum.
+// Footprint of target point X in source camera u.  K = 4: the bilinear
+// footprint around the projection (TL corner i0, j0 and the weight factors
+// ax = (1-fx, fx), ay = (1-fy, fy)); K = 1: the token (i0, j0) containing
+// the projection.  Returns false when no tap can be inside the image.
+struct Footprint {
+    int i0, j0;
+    float ax[2], ay[2];
+};
+
 template <int K>
-__device__ __forceinline__ void compute_taps(const geocache_camera& cam, const float* __restrict__ pos_u,
-                                             const uint8_t* __restrict__ valid_u, int H, int W,
-                                             float X0, float X1, float X2, float tau2, Taps& t) {
-    taps_clear(t);
+__device__ __forceinline__ bool footprint(const geocache_camera& cam, float X0, float X1, float X2, int H, int W,
+                                          Footprint& f) {
     float uu, vv;
-    if (!project(cam, X0, X1, X2, uu, vv)) return;
+    if (!project(cam, X0, X1, X2, uu, vv)) return false;
     if (K == 1) {
-        if (!(uu >= 0.0f && uu < (float)W && vv >= 0.0f && vv < (float)H)) return;
-        const int col = (int)floorf(uu), row = (int)floorf(vv);
+        if (!(uu >= 0.0f && uu < (float)W && vv >= 0.0f && vv < (float)H)) return false;
+        f.i0 = (int)floorf(uu);
+        f.j0 = (int)floorf(vv);
+        f.ax[0] = f.ax[1] = f.ay[0] = f.ay[1] = 1.0f;
+        return true;
+    }
+    const float x = __fsub_rn(uu, 0.5f), y = __fsub_rn(vv, 0.5f);
+    if (!(x >= -1.0f && x < (float)W && y >= -1.0f && y < (float)H)) return false;
+    const float i0f = floorf(x), j0f = floorf(y);
+    f.i0 = (int)i0f;
+    f.j0 = (int)j0f;
+    const float fx = __fsub_rn(x, i0f), fy = __fsub_rn(y, j0f);
+    f.ax[0] = __fsub_rn(1.0f, fx);
+    f.ax[1] = fx;
+    f.ay[0] = __fsub_rn(1.0f, fy);
+    f.ay[1] = fy;
+    return true;
+}
+
+// Per-tap tests: inside the image, non-zero weight factors, foreground
+// texel, ||P_u(q) - X||^2 <= tau2.  Returns the keep mask (bit k = tap k,
+// taps ordered TL, TR, BL, BR).
+template <int K>
+__device__ __forceinline__ int tap_mask(const Footprint& f, const float* __restrict__ pos_u,
+                                        const uint8_t* __restrict__ valid_u, int H, int W, float X0, float X1,
+                                        float X2, float tau2) {
+    int mask = 0;
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+        const int di = k & 1, dj = k >> 1;
+        const int col = f.i0 + di, row = f.j0 + dj;
+        if (col < 0 || col >= W || row < 0 || row >= H) continue;
+        if (K == 4 && (f.ax[di] == 0.0f || f.ay[dj] == 0.0f)) continue;
         const int q = row * W + col;
-        if (!__ldg(valid_u + q)) return;
-        if (!(sqdist(pos_u + 3 * (size_t)q, X0, X1, X2) <= tau2)) return;
-        t.q[0] = q;
+        if (!__ldg(valid_u + q)) continue;
+        if (!(sqdist(pos_u + 3 * (size_t)q, X0, X1, X2) <= tau2)) continue;
+        mask |= 1 << k;
+    }
+    return mask;
+}
+
+// Indices and renormalised weights of the kept taps of a footprint.
+template <int K>
+__device__ __forceinline__ void taps_from_mask(const Footprint& f, int mask, int W, Taps& t) {
+    taps_clear(t);
+    if (!mask) return;
+    if (K == 1) {
+        t.q[0] = f.j0 * W + f.i0;
         t.w[0] = 1.0f;
         t.kept = 1;
         return;
-    } else {
-        const float x = __fsub_rn(uu, 0.5f), y = __fsub_rn(vv, 0.5f);
-        if (!(x >= -1.0f && x < (float)W && y >= -1.0f && y < (float)H)) return;
-        const float i0f = floorf(x), j0f = floorf(y);
-        const int i0 = (int)i0f, j0 = (int)j0f;
-        const float fx = __fsub_rn(x, i0f), fy = __fsub_rn(y, j0f);
-        const float ax[2] = {__fsub_rn(1.0f, fx), fx};
-        const float ay[2] = {__fsub_rn(1.0f, fy), fy};
-        float raw[4];
-        float sum = 0.0f;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int di = k & 1, dj = k >> 1;
-            const int col = i0 + di, row = j0 + dj;
-            raw[k] = 0.0f;
-            if (col < 0 || col >= W || row < 0 || row >= H) continue;
-            if (ax[di] == 0.0f || ay[dj] == 0.0f) continue;
-            const int q = row * W + col;
-            if (!__ldg(valid_u + q)) continue;
-            if (!(sqdist(pos_u + 3 * (size_t)q, X0, X1, X2) <= tau2)) continue;
-            raw[k] = __fmul_rn(ax[di], ay[dj]);
-            t.q[k] = q;
-            sum = __fadd_rn(sum, raw[k]);
-            ++t.kept;
-        }
-        if (t.kept) {
-#pragma unroll
-            for (int k = 0; k < 4; ++k)
-                if (t.q[k] >= 0) t.w[k] = __fdiv_rn(raw[k], sum);
-        }
     }
+    float raw[4];
+    float sum = 0.0f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        raw[k] = 0.0f;
+        if (!((mask >> k) & 1)) continue;
+        const int di = k & 1, dj = k >> 1;
+        raw[k] = __fmul_rn(f.ax[di], f.ay[dj]);
+        t.q[k] = (f.j0 + dj) * W + (f.i0 + di);
+        sum = __fadd_rn(sum, raw[k]);
+        ++t.kept;
+    }
+    const float rs = __frcp_rn(sum);
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+        if (t.q[k] >= 0) t.w[k] = __fmul_rn(raw[k], rs);
+}
+
+// Taps of target point X in source view u (pos_u [H*W*3], valid_u [H*W]):
+// footprint, per-tap tests, renormalised weights.  *mask_out (optional)
+// receives the keep mask.
+template <int K>
+__device__ __forceinline__ void compute_taps(const geocache_camera& cam, const float* __restrict__ pos_u,
+                                             const uint8_t* __restrict__ valid_u, int H, int W,
+                                             float X0, float X1, float X2, float tau2, Taps& t,
+                                             int* mask_out = nullptr) {
+    Footprint f;
+    int mask = 0;
+    if (footprint<K>(cam, X0, X1, X2, H, W, f)) mask = tap_mask<K>(f, pos_u, valid_u, H, W, X0, X1, X2, tau2);
+    taps_from_mask<K>(f, mask, W, t);
+    if (mask_out) *mask_out = mask;
 }
 
 }  // namespace geocache

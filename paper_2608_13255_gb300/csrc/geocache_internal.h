@@ -31,6 +31,7 @@ struct TransportArgs {
     const float* tau;
     const int32_t* idx;
     const float* w;
+    const uint8_t* keep;
     const float* x0_new;
     const float* x0_prev;
     float* x0_out;
@@ -46,6 +47,7 @@ cudaError_t launch_tau(const float* pos, const uint8_t* valid, int B, int N, int
                        float tol_frac, float* tau, cudaStream_t s);
 cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s);
 cudaError_t launch_transport(const TransportArgs& t, cudaStream_t s);
+int transport_launch_count(int a, int C, int in_place);
 cudaError_t launch_copy_anchor_rows(const TransportArgs& t, cudaStream_t s);
 cudaError_t launch_reconstruct(const void* x_t, const float* x0, void* x_next, int lat_dtype, int64_t n,
                                const ReconCoef& coef, float* pred_out, float* x0_store, cudaStream_t s);

@@ -20,7 +20,7 @@ OK, EINVAL, ESHAPE, EDTYPE, ECUDA, ETIMEOUT, EDEVICE, EALIAS = 0, -1, -2, -3, -4
 F32, BF16 = 0, 1
 DDIM, FM_EULER = 0, 1
 PRED_NONE, PRED_EPS, PRED_V, PRED_VELOCITY = 0, 1, 2, 3
-CORR_GEOMETRY, CORR_TABLE = 0, 1
+CORR_GEOMETRY, CORR_TABLE, CORR_MASK = 0, 1, 2
 SCHED_EVERY_K, SCHED_HEAD_MID_TAIL, SCHED_LIST, SCHED_ALL_FULL, SCHED_SINGLE_CACHED = 0, 1, 2, 3, 4
 MAX_VIEWS = 64
 
@@ -45,7 +45,7 @@ class Corr(ctypes.Structure):
                 ("K", ctypes.c_int), ("tol_frac", ctypes.c_float),
                 ("pos", ctypes.c_void_p), ("valid", ctypes.c_void_p), ("cams", ctypes.c_void_p),
                 ("tau", ctypes.c_void_p), ("idx", ctypes.c_void_p), ("w", ctypes.c_void_p),
-                ("mode", ctypes.c_int)]
+                ("keep", ctypes.c_void_p), ("mode", ctypes.c_int)]
 
 
 class Recon(ctypes.Structure):
@@ -159,18 +159,26 @@ class CorrHandle:
     def w(self):
         return self._keep.get("w")
 
+    @property
+    def keep(self):
+        return self._keep.get("keep")
 
-def make_corr(pos, valid, cams, tau, idx=None, w=None, K=4, tol_frac=0.01, mode=None) -> CorrHandle:
-    """Describe a batch's geometry (and optional tables) for the C ABI."""
+
+def make_corr(pos, valid, cams, tau, idx=None, w=None, K=4, tol_frac=0.01, mode=None, keep=None) -> CorrHandle:
+    """Describe a batch's geometry (and optional tables / keep masks) for the
+    C ABI.  The default mode is MASK when keep masks are given, else TABLE
+    when tables are given, else GEOMETRY."""
     B, N, H, W = valid.shape
     n = B * N * H * W
-    keep = {"pos": pos, "valid": valid, "cams": cams, "tau": tau, "idx": idx, "w": w}
+    refs = {"pos": pos, "valid": valid, "cams": cams, "tau": tau, "idx": idx, "w": w, "keep": keep}
+    if mode is None:
+        mode = CORR_MASK if keep is not None else (CORR_TABLE if idx is not None else CORR_GEOMETRY)
     c = Corr(B, N, H, W, K, tol_frac,
              _dev(pos, torch.float32, 3 * n, "pos"), _dev(valid, torch.uint8, n, "valid"),
              _dev(cams, torch.float32, 16 * B * N, "cams"), _dev(tau, torch.float32, B, "tau"),
              _dev(idx, torch.int32, n * N * K, "idx"), _dev(w, torch.float32, n * N * K, "w"),
-             (CORR_TABLE if idx is not None else CORR_GEOMETRY) if mode is None else mode)
-    return CorrHandle(c, keep)
+             _dev(keep, torch.uint8, n * N, "keep"), mode)
+    return CorrHandle(c, refs)
 
 
 def make_recon(sampler="ddim", a_t=0.0, a_prev=0.0, sigma=0.0, sigma_next=0.0, pred_kind=None,
@@ -256,6 +264,14 @@ def rotate_anchors(N: int, a: int, step: int, S: int, sched: dict):
     _check(load().geocache_rotate_anchors(int(N), int(a), int(step), int(S), ctypes.byref(s),
                                           ctypes.cast(out, ctypes.c_void_p), ctypes.byref(full)))
     return list(out), bool(full.value)
+
+
+def transport_launches(a: int, C: int, in_place: bool = False) -> int:
+    """Kernels one geocache_transport_step enqueues: the tiled kernel for
+    a <= 8 anchors (else one per group of 16 channels), plus the anchor-row
+    copy of an in-place update."""
+    n = 1 if a <= 8 else -(-C // (4 if C <= 4 else 16))
+    return n + (1 if in_place else 0)
 
 
 def abi_version() -> int:

@@ -107,11 +107,15 @@ def pred_scale(params):
 
 
 class DeviceGeometry:
-    """A workload's geometry on the GPU, with tau and (optionally) tables."""
+    """A workload's geometry on the GPU, with tau, the keep masks and
+    (optionally) the idx/w tables, built by geocache_build_corr.  `corr`
+    uses the keep masks (the fast path); corr_for(mode) gives the others."""
 
     def __init__(self, w, K=4, tables=True, dev="cuda"):
         from paper_2608_13255_gb300 import geocache as gc
+        self.gc = gc
         self.w = w
+        self.K = K
         self.pos = torch.from_numpy(w.pos).to(dev)
         self.valid = torch.from_numpy(w.valid).to(dev)
         self.cams = torch.from_numpy(w.cams).to(dev)
@@ -121,6 +125,13 @@ class DeviceGeometry:
             shp = (w.B, w.N, w.N, w.H, w.W, K)
             self.idx = torch.empty(shp, dtype=torch.int32, device=dev)
             self.wt = torch.empty(shp, dtype=torch.float32, device=dev)
+        self.keep = torch.empty((w.B, w.N, w.N, w.H, w.W), dtype=torch.uint8, device=dev)
         self.corr = gc.make_corr(self.pos, self.valid, self.cams, self.tau, self.idx, self.wt, K=K,
-                                 tol_frac=w.tol_frac, mode=gc.CORR_GEOMETRY)
+                                 tol_frac=w.tol_frac, keep=self.keep, mode=gc.CORR_MASK)
         gc.build_corr(self.corr)
+
+    def corr_for(self, mode):
+        gc = self.gc
+        m = {"mask": gc.CORR_MASK, "geometry": gc.CORR_GEOMETRY, "table": gc.CORR_TABLE}[mode]
+        return gc.make_corr(self.pos, self.valid, self.cams, self.tau, self.idx, self.wt, K=self.K,
+                            tol_frac=self.w.tol_frac, keep=self.keep, mode=m)

@@ -79,7 +79,7 @@ def test_argument_errors_before_launch(gc):
     # NULL corr, bad sizes, bad anchors, bad sampler: rejected on the host
     assert L.geocache_transport_step(None, None, 0, 0, None, None, None, None, None, 0, None, None) == gc.EINVAL
     assert "corr" in gc.last_error()
-    c = gc.Corr(1, 6, 8, 8, 4, 0.01, 16, 16, 16, 16, None, None, gc.CORR_GEOMETRY)
+    c = gc.Corr(1, 6, 8, 8, 4, 0.01, 16, 16, 16, 16, None, None, None, gc.CORR_GEOMETRY)
     anc = (ctypes.c_int32 * 2)(3, 0)  # not ascending
     st = L.geocache_transport_step(ctypes.byref(c), ctypes.cast(anc, ctypes.c_void_p), 2, 4, 16, 16, 32,
                                    None, None, 0, None, None)
@@ -93,6 +93,11 @@ def test_argument_errors_before_launch(gc):
                                    None, None, 0, None, None)
     assert st == gc.EINVAL
     c.K = 4
+    c.mode = gc.CORR_MASK  # mask mode without keep masks
+    st = L.geocache_transport_step(ctypes.byref(c), ctypes.cast(anc, ctypes.c_void_p), 2, 4, 16, 16, 32,
+                                   None, None, 0, None, None)
+    assert st == gc.EINVAL and "keep" in gc.last_error()
+    c.mode = gc.CORR_GEOMETRY
     c.N = 65
     assert L.geocache_build_corr(ctypes.byref(c), None) == gc.ESHAPE
     c.N = 6

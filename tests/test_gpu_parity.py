@@ -43,6 +43,10 @@ def _compare_tables(w, g, K):
     assert not mism.any(), "%d index mismatches outside the threshold band" % mism.sum()
     kept = idx_ref >= 0
     assert_f32_close(wt[~inband], w_ref[~inband], what="weights")
+    # keep masks: bit k set iff tap k is kept
+    keep_ref = sum((kept[..., k].astype(np.uint8) << k) for k in range(K))
+    keep = g.keep.cpu().numpy()
+    assert not ((keep != keep_ref) & (band == 0)).any(), "keep masks differ outside the threshold band"
     return int(band.sum()), float(kept.any(-1).mean())
 
 
@@ -63,7 +67,7 @@ def test_tables_bit_exact_k1(gc, workloads, name):
     _compare_tables(w, g, 1)
 
 
-def _run_step(gc, w, g, anchors, params, pred=None, mode="geometry", inplace=False, xinplace=False,
+def _run_step(gc, w, g, anchors, params, pred=None, mode="mask", inplace=False, xinplace=False,
               seed_extra=0, C=None):
     """One cached step on the GPU and in the oracle from the same inputs."""
     if C is not None and C != w.C:
@@ -77,9 +81,7 @@ def _run_step(gc, w, g, anchors, params, pred=None, mode="geometry", inplace=Fal
     d_xt = xt_t.to(dev)
     d_xn = d_xt if xinplace else torch.empty_like(d_xt)
     d_pred = torch.empty_like(d_prev) if pred else None
-    corr = g.corr
-    if mode == "table":
-        corr = gc.make_corr(g.pos, g.valid, g.cams, g.tau, g.idx, g.wt, K=g.corr.c.K, mode=gc.CORR_TABLE)
+    corr = g.corr_for(mode)
     r = gc.make_recon(params["sampler"], a_t=params.get("a_t", 0), a_prev=params.get("a_prev", 0),
                       sigma=params.get("sigma", 0), sigma_next=params.get("sigma_next", 0),
                       pred_kind=pred, pred_out=d_pred)
@@ -125,15 +127,18 @@ def test_transport_step_parity(gc, workloads, name):
     print("%s anchors %s: max |dx0| %.3g, max |dx_next| %.3g" % (name, anchors, e0, e1))
 
 
-@pytest.mark.parametrize("name", ["hunyuan64", "ring12_128"])
-def test_transport_table_mode_matches_geometry_mode(gc, workloads, name):
+@pytest.mark.parametrize("name,K", [("hunyuan64", 4), ("ring12_128", 4), ("solids96", 1)])
+def test_corr_modes_agree_bitwise(gc, workloads, name, K):
+    # keep masks, full geometry and tables give the same taps and weights
     w = workloads(name)
-    g = DeviceGeometry(w, K=w.K)
+    g = DeviceGeometry(w, K=K)
     anchors = oracle.rotate_anchors(w.N, w.a, 1)
     params = synth.recon_params(w, 7)
+    _, _, got_mask, _ = _run_step(gc, w, g, anchors, params, mode="mask")
     _, _, got_geom, _ = _run_step(gc, w, g, anchors, params, mode="geometry")
     _, _, got_tab, _ = _run_step(gc, w, g, anchors, params, mode="table")
-    np.testing.assert_array_equal(got_geom, got_tab)  # same taps, same arithmetic
+    np.testing.assert_array_equal(got_mask, got_geom)
+    np.testing.assert_array_equal(got_mask, got_tab)
 
 
 @pytest.mark.parametrize("pred", ["eps", "v"])
@@ -193,6 +198,9 @@ def test_ragged_tiles_and_many_views(gc):
     torch.cuda.synchronize()
     _compare_tables(wv, g, 4)
     _run_step(gc, wv, g, oracle.rotate_anchors(64, 8, 3), synth.recon_params(wv, 0))
+    # more anchors than the tiled kernel holds (general per-token kernel), K = 4 and K = 1
+    _run_step(gc, wv, g, oracle.rotate_anchors(64, 12, 1), synth.recon_params(wv, 0))
+    _run_step(gc, wv, g, oracle.rotate_anchors(64, 12, 1), synth.recon_params(wv, 0), mode="table")
 
 
 def test_empty_asset_keeps_state(gc, workloads):
@@ -212,7 +220,7 @@ def test_empty_asset_keeps_state(gc, workloads):
 def test_zero_delta_bit_identical(gc, workloads):
     w = workloads("ring12_128")
     g = DeviceGeometry(w, K=4, tables=False)
-    x0_prev, _, _ = step_inputs(w, 3, [0, 3, 6, 9])
+    x0_prev, _, _ = step_inputs(w, 3, [0, 3, 6, 9])  # keep-mask path
     d_prev = torch.from_numpy(x0_prev).cuda()
     d_new = d_prev[:, [0, 3, 6, 9]].contiguous()
     d_out = torch.empty_like(d_prev)
