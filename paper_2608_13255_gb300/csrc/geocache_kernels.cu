@@ -166,127 +166,35 @@ cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s) {
 }
 
 // ------------------------------------------------- fused transport step --
-// General variant (any number of anchors): one thread per (asset b, view v,
-// token p), channels [c0, c0+cn) with cn <= CMAX.  Anchor views take the
-// denoiser's x0; other views add the mean over covering anchors of the
-// tap-weighted anchor increments (Eq. 1), then every view is reconstructed
-// (Sec. 3.2).
-template <typename T, int K, int CMAX>
-__global__ void __launch_bounds__(256) transport_pixel_kernel(const TransportArgs args) {
-    const int HW = args.H * args.W;
-    const int p = blockIdx.x * blockDim.x + threadIdx.x;
-    const int v = blockIdx.y, b = blockIdx.z;
-    if (p >= HW) return;
-    const int N = args.N, C = args.C, cn = args.cn, c0 = args.c0;
-    const size_t plane0 = (((size_t)b * N + v) * C + c0) * HW + p;  // element (b, v, c0, p)
-    const int slot = args.slot_of[v];
-    float x0v[CMAX];
-    if (slot >= 0) {
-        const float* src = args.x0_new + (((size_t)b * args.a + slot) * C + c0) * HW + p;
-#pragma unroll
-        for (int c = 0; c < CMAX; ++c)
-            if (c < cn) x0v[c] = __ldg(src + (size_t)c * HW);
-        if (args.write_anchor_rows) {
-#pragma unroll
-            for (int c = 0; c < CMAX; ++c)
-                if (c < cn) args.x0_out[plane0 + (size_t)c * HW] = x0v[c];
-        }
-    } else {
-        float acc[CMAX];
-#pragma unroll
-        for (int c = 0; c < CMAX; ++c) acc[c] = 0.0f;
-        int n = 0;
-        const size_t tv = ((size_t)b * N + v) * HW + p;
-        const bool fg = (args.mode == GEOCACHE_CORR_TABLE) || __ldg(args.valid + tv);
-        float X0 = 0.f, X1 = 0.f, X2 = 0.f, tau2 = 0.f;
-        if (fg && args.mode != GEOCACHE_CORR_TABLE) {  // geometry and keep-mask modes recompute the taps
-            X0 = __ldg(args.pos + 3 * tv);
-            X1 = __ldg(args.pos + 3 * tv + 1);
-            X2 = __ldg(args.pos + 3 * tv + 2);
-            const float tu = __ldg(args.tau + b);
-            tau2 = __fmul_rn(tu, tu);
-        }
-        if (fg) {
-            for (int s = 0; s < args.a; ++s) {
-                const int u = args.anchors[s];
-                Taps t;
-                if (args.mode == GEOCACHE_CORR_TABLE) {
-                    const size_t row = (((size_t)b * N + v) * N + u) * HW + p;
-                    t.kept = 0;
-#pragma unroll
-                    for (int k = 0; k < K; ++k) {
-                        t.q[k] = __ldg(args.idx + row * K + k);
-                        t.w[k] = __ldg(args.w + row * K + k);
-                        t.kept += t.q[k] >= 0;
-                    }
-                } else {
-                    const size_t su = ((size_t)b * N + u) * HW;
-                    compute_taps<K>(args.cams[(size_t)b * N + u], args.pos + 3 * su, args.valid + su,
-                                    args.H, args.W, X0, X1, X2, tau2, t);
-                }
-                if (!t.kept) continue;
-                ++n;
-                const float* xn = args.x0_new + (((size_t)b * args.a + s) * C + c0) * HW;
-                const float* xp = args.x0_prev + (((size_t)b * N + u) * C + c0) * HW;
-#pragma unroll
-                for (int c = 0; c < CMAX; ++c) {
-                    if (c >= cn) break;
-                    float g = 0.0f;
-#pragma unroll
-                    for (int k = 0; k < K; ++k) {
-                        if (t.q[k] < 0) continue;
-                        const size_t e = (size_t)c * HW + t.q[k];
-                        g = __fmaf_rn(t.w[k], __fsub_rn(__ldg(xn + e), __ldg(xp + e)), g);
-                    }
-                    acc[c] = __fadd_rn(acc[c], g);
-                }
-            }
-        }
-#pragma unroll
-        for (int c = 0; c < CMAX; ++c) {
-            if (c < cn) {
-                const float prev = __ldg(args.x0_prev + plane0 + (size_t)c * HW);
-                x0v[c] = n ? __fadd_rn(prev, __fdiv_rn(acc[c], (float)n)) : prev;
-                args.x0_out[plane0 + (size_t)c * HW] = x0v[c];
-            }
-        }
-    }
-    if (args.coef.enabled) {
-        const T* xt = static_cast<const T*>(args.x_t);
-        T* xnx = static_cast<T*>(args.x_next);
-#pragma unroll
-        for (int c = 0; c < CMAX; ++c) {
-            if (c < cn) {
-                const size_t e = plane0 + (size_t)c * HW;
-                float pred;
-                const float y = recon_one(args.coef, lat_load(xt, e), x0v[c], pred);
-                lat_store(xnx, e, y);
-                if (args.pred_out) args.pred_out[e] = pred;
-            }
-        }
-    }
-}
-
-// Tiled variant (a <= kTileMaxAnchors), the hot path.  One CTA owns a tile
-// of 256 consecutive tokens of one view (asset b, view v) and all channels.
-//  phase 0 (views outside the anchor set): thread t finds the kept taps of
-//    token 4*(t%64) + t/64 for every anchor and stores them in shared memory
-//    at column t, with the number n of covering anchors;
-//  phase 1: thread t handles the 4 consecutive tokens 4*(t%64).. of channel
-//    t/64 (+4, +8, ... for C > 4): 16-byte loads of x0(t-1) or the anchor's
-//    x0 and of x_t (issued before phase 0 so they overlap the geometry), the
-//    gathered increment sum_j w_j (x0_new - x0_prev)[q_j] / n, the cache
-//    store and the sampler reconstruction.
-// Streamed rows use evict-first cache hints so that the anchors' rows, which
-// the gathers re-read, stay in L2.
-constexpr int kTile = 256;
-constexpr int kTileMaxAnchors = 8;
+// One thread per quad of 4 consecutive tokens of one view (asset b, view v),
+// all channels in groups of 4.  For each group the thread issues 16-byte
+// loads of x0 (the anchor's fresh x0, or x0(t-1)) and of x_t first, then for
+// views outside the anchor set adds to each covered token the mean over the
+// covering anchors of the tap-weighted anchor increments (Eq. 1 with the
+// multi-anchor aggregation of Sec. 3.2; uncovered tokens keep x0(t-1)), then
+// stores x0(t) and the sampler reconstruction of every token.
+// Taps come from the keep masks (MODE = GEOCACHE_CORR_MASK: projection and
+// weights recomputed only for covered (token, anchor) pairs), from the full
+// per-tap tests (GEOMETRY) or from the tables (TABLE); all three are
+// bit-identical.  Streamed rows use evict-first hints so that the anchors'
+// rows, which the gathers re-read, stay in L2.
+constexpr int kThreads = 256;
 
 template <typename T>
 struct Lat4;
 template <>
 struct Lat4<float> {
-    using V = float4;
+    using Raw = float4;
+    __device__ static Raw load_raw(const float* p, size_t e, int cnt, bool vec) {
+        if (vec) return __ldcs(reinterpret_cast<const float4*>(p + e));
+        float4 r = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (cnt > 0) r.x = __ldcs(p + e);
+        if (cnt > 1) r.y = __ldcs(p + e + 1);
+        if (cnt > 2) r.z = __ldcs(p + e + 2);
+        if (cnt > 3) r.w = __ldcs(p + e + 3);
+        return r;
+    }
+    __device__ static void unpack(const Raw& x, float (&r)[4]) { r[0] = x.x; r[1] = x.y; r[2] = x.z; r[3] = x.w; }
     __device__ static void load(const float* p, size_t e, int cnt, bool vec, float (&r)[4]) {
         if (vec) {
             const float4 x = __ldcs(reinterpret_cast<const float4*>(p + e));
@@ -308,6 +216,22 @@ struct Lat4<float> {
 };
 template <>
 struct Lat4<__nv_bfloat16> {
+    using Raw = uint2;
+    __device__ static Raw load_raw(const __nv_bfloat16* p, size_t e, int cnt, bool vec) {
+        if (vec) return __ldcs(reinterpret_cast<const uint2*>(p + e));
+        const unsigned short* q = reinterpret_cast<const unsigned short*>(p + e);
+        uint32_t h[4] = {0, 0, 0, 0};
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            if (i < cnt) h[i] = q[i];
+        return make_uint2(h[0] | (h[1] << 16), h[2] | (h[3] << 16));
+    }
+    __device__ static void unpack(const Raw& x, float (&r)[4]) {
+        r[0] = __uint_as_float(x.x << 16);
+        r[1] = __uint_as_float(x.x & 0xffff0000u);
+        r[2] = __uint_as_float(x.y << 16);
+        r[3] = __uint_as_float(x.y & 0xffff0000u);
+    }
     __device__ static void load(const __nv_bfloat16* p, size_t e, int cnt, bool vec, float (&r)[4]) {
         if (vec) {
             const uint2 x = __ldcs(reinterpret_cast<const uint2*>(p + e));
@@ -335,10 +259,7 @@ struct Lat4<__nv_bfloat16> {
     }
 };
 
-__device__ __forceinline__ void f4_load(const float* p, size_t e, int cnt, bool vec, float (&r)[4]) {
-    Lat4<float>::load(p, e, cnt, vec, r);
-}
-// anchor rows: keep them in L2 for the gathers (default caching)
+// the anchors' rows stay cached (they are re-read by the gathers)
 __device__ __forceinline__ void f4_load_keep(const float* p, size_t e, int cnt, bool vec, float (&r)[4]) {
     if (vec) {
         const float4 x = __ldg(reinterpret_cast<const float4*>(p + e));
@@ -349,210 +270,182 @@ __device__ __forceinline__ void f4_load_keep(const float* p, size_t e, int cnt, 
     }
 }
 
-template <typename T, int K, bool VEC>
-__global__ void __launch_bounds__(kTile) transport_tile_kernel(const TransportArgs args) {
-    extern __shared__ __align__(16) unsigned char smem[];
+// Keep masks of the quad's tokens for source view u, one byte per token.
+__device__ __forceinline__ uint32_t quad_masks(const uint8_t* row, int cnt, bool vec) {
+    if (vec) return __ldg(reinterpret_cast<const uint32_t*>(row));
+    uint32_t m = 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        if (i < cnt) m |= (uint32_t)__ldg(row + i) << (8 * i);
+    return m;
+}
+
+template <typename T, int K, int MODE, bool VEC>
+__global__ void __launch_bounds__(kThreads) transport_quad_kernel(const TransportArgs args) {
     const int HW = args.H * args.W;
-    const int tile0 = blockIdx.x * kTile;
+    const int p0 = 4 * (blockIdx.x * kThreads + threadIdx.x);
+    if (p0 >= HW) return;
+    const int cnt = HW - p0 < 4 ? HW - p0 : 4;
     const int v = blockIdx.y, b = blockIdx.z;
     const int N = args.N, C = args.C, a = args.a;
     const int slot = args.slot_of[v];
-    const int t = threadIdx.x;
-    const int quad = t & 63;
-    const int E = K * a;  // tap entries per token
-    geocache_camera* s_cam = reinterpret_cast<geocache_camera*>(smem);
-    int32_t* s_q = reinterpret_cast<int32_t*>(smem + sizeof(geocache_camera) * kTileMaxAnchors);
-    float* s_w = reinterpret_cast<float*>(s_q + E * kTile);
-    uint8_t* s_s = reinterpret_cast<uint8_t*>(s_w + E * kTile);
-    uint8_t* s_len = s_s + E * kTile;
-    uint8_t* s_n = s_len + kTile;
-
-    // phase-1 role and the first channel pass's streaming loads
-    const int p0 = tile0 + 4 * quad;
-    const int cnt = HW - p0 < 4 ? HW - p0 : 4;
-    int c = t >> 6;
-    const size_t view_base = ((size_t)b * N + v) * C;
-    const size_t anc_base = slot >= 0 ? ((size_t)b * a + slot) * C : 0;
+    const size_t plane = (size_t)HW;
+    const size_t view_base = ((size_t)b * N + v) * C * plane + p0;   // element (b, v, 0, p0)
     const bool recon = args.coef.enabled;
     const T* xt_p = static_cast<const T*>(args.x_t);
-    float x0[4], xt[4];
-    if (cnt > 0 && c < C) {
-        if (slot >= 0)
-            f4_load_keep(args.x0_new, (anc_base + c) * HW + p0, cnt, VEC, x0);
-        else
-            f4_load(args.x0_prev, (view_base + c) * HW + p0, cnt, VEC, x0);
-        if (recon) Lat4<T>::load(xt_p, (view_base + c) * HW + p0, cnt, VEC, xt);
+    T* xn_p = static_cast<T*>(args.x_next);
+    const size_t tv = ((size_t)b * N + v) * plane + p0;              // token p0 of (b, v)
+
+    // which of the quad's tokens have any kept tap (any anchor)
+    uint32_t any_cover = 0;
+    float tau2 = 0.0f;
+    if (slot < 0) {
+        if (MODE == GEOCACHE_CORR_MASK) {
+            const uint8_t* krow = args.keep + ((size_t)b * N + v) * N * plane + p0;
+            for (int s = 0; s < a; ++s) any_cover |= quad_masks(krow + (size_t)args.anchors[s] * plane, cnt, VEC);
+        } else if (MODE == GEOCACHE_CORR_GEOMETRY) {
+            any_cover = quad_masks(args.valid + tv, cnt, VEC);
+            const float tu = __ldg(args.tau + b);
+            tau2 = __fmul_rn(tu, tu);
+        } else {
+            any_cover = 0x01010101u;  // tables: every token is looked up
+        }
     }
 
-    if (slot < 0) {
-        // ------------------------------------------------------ phase 0 --
-        const bool table = args.mode == GEOCACHE_CORR_TABLE;
-        if (!table)
-            for (int i = t; i < a * 16; i += kTile)
-                reinterpret_cast<float*>(s_cam)[i] =
-                    __ldg(reinterpret_cast<const float*>(args.cams + (size_t)b * N + args.anchors[i >> 4]) + (i & 15));
-        __syncthreads();
-        const int p = tile0 + 4 * (t & 63) + (t >> 6);
-        int len = 0, n = 0;
-        if (p < HW) {
-            const size_t tv = ((size_t)b * N + v) * HW + p;
-            if (table) {
-                for (int s = 0; s < a; ++s) {
-                    const size_t row = (((size_t)b * N + v) * N + args.anchors[s]) * HW + p;
-                    int kept = 0;
+    for (int cg = 0; cg < C; cg += 4) {
+        const int cn = C - cg < 4 ? C - cg : 4;
+        float x0[4][4];
+        typename Lat4<T>::Raw xt[4];
+        // streaming loads of the channel group first
 #pragma unroll
-                    for (int k = 0; k < K; ++k) {
-                        const int32_t q = __ldg(args.idx + row * K + k);
-                        if (q >= 0) {
-                            s_q[len * kTile + t] = q;
-                            s_w[len * kTile + t] = __ldg(args.w + row * K + k);
-                            s_s[len * kTile + t] = (uint8_t)s;
-                            ++len;
-                            ++kept;
-                        }
+        for (int c = 0; c < 4; ++c) {
+            if (c >= cn) break;
+            const size_t e = view_base + (size_t)(cg + c) * plane;
+            if (slot >= 0)
+                f4_load_keep(args.x0_new, (((size_t)b * a + slot) * C + cg + c) * plane + p0, cnt, VEC, x0[c]);
+            else
+                Lat4<float>::load(args.x0_prev, e, cnt, VEC, x0[c]);
+            if (recon) xt[c] = Lat4<T>::load_raw(xt_p, e, cnt, VEC);
+        }
+        if (slot < 0) {
+            if (any_cover) {
+#pragma unroll 1
+                for (int i = 0; i < 4; ++i) {
+                    if (!((any_cover >> (8 * i)) & 0xff)) continue;
+                    const int p = p0 + i;
+                    float X0 = 0.f, X1 = 0.f, X2 = 0.f;
+                    if (MODE != GEOCACHE_CORR_TABLE) {
+                        X0 = __ldg(args.pos + 3 * (tv + i));
+                        X1 = __ldg(args.pos + 3 * (tv + i) + 1);
+                        X2 = __ldg(args.pos + 3 * (tv + i) + 2);
                     }
-                    n += kept > 0;
-                }
-            } else if (args.mode == GEOCACHE_CORR_MASK) {
-                // keep masks of every anchor first (independent byte loads), then
-                // the projection and weights only for the covering anchors
-                const uint8_t* krow = args.keep + ((size_t)b * N + v) * N * HW + p;
-                uint32_t masks = 0;
-                for (int s = 0; s < a; ++s) masks |= (uint32_t)__ldg(krow + (size_t)args.anchors[s] * HW) << (4 * s);
-                if (masks) {
-                    const float X0 = __ldg(args.pos + 3 * tv), X1 = __ldg(args.pos + 3 * tv + 1),
-                                X2 = __ldg(args.pos + 3 * tv + 2);
+                    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+                    int n = 0;
                     for (int s = 0; s < a; ++s) {
-                        const int m = (masks >> (4 * s)) & 15;
-                        if (!m) continue;
-                        Footprint f;
-                        footprint<K>(s_cam[s], X0, X1, X2, args.H, args.W, f);
+                        const int u = args.anchors[s];
                         Taps tp;
-                        taps_from_mask<K>(f, m, args.W, tp);
+                        if (MODE == GEOCACHE_CORR_TABLE) {
+                            const size_t row = (((size_t)b * N + v) * N + u) * plane + p;
+                            tp.kept = 0;
+#pragma unroll
+                            for (int k = 0; k < K; ++k) {
+                                tp.q[k] = __ldg(args.idx + row * K + k);
+                                tp.w[k] = __ldg(args.w + row * K + k);
+                                tp.kept += tp.q[k] >= 0;
+                            }
+                        } else {
+                            const geocache_camera& cam = args.cams[(size_t)b * N + u];
+                            if (MODE == GEOCACHE_CORR_MASK) {
+                                const int m = __ldg(args.keep + (((size_t)b * N + v) * N + u) * plane + p);
+                                if (!m) continue;
+                                Footprint f;
+                                footprint<K>(cam, X0, X1, X2, args.H, args.W, f);
+                                taps_from_mask<K>(f, m, args.W, tp);
+                            } else {
+                                const size_t su = ((size_t)b * N + u) * plane;
+                                compute_taps<K>(cam, args.pos + 3 * su, args.valid + su, args.H, args.W, X0, X1, X2,
+                                                tau2, tp);
+                            }
+                        }
+                        if (!tp.kept) continue;
                         ++n;
+                        const float* xn = args.x0_new + (((size_t)b * a + s) * C + cg) * plane;
+                        const float* xp = args.x0_prev + (((size_t)b * N + u) * C + cg) * plane;
 #pragma unroll
                         for (int k = 0; k < K; ++k) {
                             if (tp.q[k] < 0) continue;
-                            s_q[len * kTile + t] = tp.q[k];
-                            s_w[len * kTile + t] = tp.w[k];
-                            s_s[len * kTile + t] = (uint8_t)s;
-                            ++len;
+#pragma unroll
+                            for (int c = 0; c < 4; ++c) {
+                                if (c >= cn) break;
+                                const size_t e = (size_t)c * plane + tp.q[k];
+                                acc[c] = __fmaf_rn(tp.w[k], __fsub_rn(__ldg(xn + e), __ldg(xp + e)), acc[c]);
+                            }
+                        }
+                    }
+                    if (n) {
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            const float g = n == 1 ? acc[c] : __fdiv_rn(acc[c], (float)n);
+#pragma unroll
+                            for (int ii = 0; ii < 4; ++ii)
+                                if (ii == i) x0[c][ii] = __fadd_rn(x0[c][ii], g);
                         }
                     }
                 }
-            } else if (__ldg(args.valid + tv)) {
-                const float X0 = __ldg(args.pos + 3 * tv), X1 = __ldg(args.pos + 3 * tv + 1),
-                            X2 = __ldg(args.pos + 3 * tv + 2);
-                const float tu = __ldg(args.tau + b);
-                const float tau2 = __fmul_rn(tu, tu);
-                for (int s = 0; s < a; ++s) {
-                    const size_t su = ((size_t)b * N + args.anchors[s]) * HW;
-                    Taps tp;
-                    compute_taps<K>(s_cam[s], args.pos + 3 * su, args.valid + su, args.H, args.W, X0, X1, X2, tau2,
-                                    tp);
-                    if (!tp.kept) continue;
-                    ++n;
-#pragma unroll
-                    for (int k = 0; k < K; ++k) {
-                        if (tp.q[k] < 0) continue;
-                        s_q[len * kTile + t] = tp.q[k];
-                        s_w[len * kTile + t] = tp.w[k];
-                        s_s[len * kTile + t] = (uint8_t)s;
-                        ++len;
-                    }
-                }
             }
-        }
-        s_len[t] = (uint8_t)len;
-        s_n[t] = (uint8_t)n;
-        __syncthreads();
-    }
-
-    // ---------------------------------------------------------- phase 1 --
-    if (cnt <= 0) return;
-    T* xn_p = static_cast<T*>(args.x_next);
-    for (; c < C; c += 4) {
-        const size_t e = (view_base + c) * HW + p0;
-        if (slot < 0) {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int col = i * 64 + quad;
-                const int n = s_n[col];
-                if (!n) continue;
-                const int len = s_len[col];
-                float acc = 0.0f;
-                for (int j = 0; j < len; ++j) {
-                    const int q = s_q[j * kTile + col];
-                    const float wj = s_w[j * kTile + col];
-                    const int s = s_s[j * kTile + col];
-                    const float xn = __ldg(args.x0_new + (((size_t)b * a + s) * C + c) * HW + q);
-                    const float xp = __ldg(args.x0_prev + (((size_t)b * N + args.anchors[s]) * C + c) * HW + q);
-                    acc = __fmaf_rn(wj, __fsub_rn(xn, xp), acc);
-                }
-                x0[i] = __fadd_rn(x0[i], __fdiv_rn(acc, (float)n));
+            for (int c = 0; c < 4; ++c) {
+                if (c >= cn) break;
+                Lat4<float>::store(args.x0_out, view_base + (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
             }
-            Lat4<float>::store(args.x0_out, e, cnt, VEC, x0);
         } else if (args.write_anchor_rows) {
-            Lat4<float>::store(args.x0_out, e, cnt, VEC, x0);
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                if (c >= cn) break;
+                Lat4<float>::store(args.x0_out, view_base + (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
+            }
         }
         if (recon) {
-            float y[4], pr[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) y[i] = recon_one(args.coef, xt[i], x0[i], pr[i]);
-            Lat4<T>::store(xn_p, e, cnt, VEC, y);
-            if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, VEC, pr);
-        }
-        if (c + 4 < C) {
-            if (slot >= 0)
-                f4_load_keep(args.x0_new, (anc_base + c + 4) * HW + p0, cnt, VEC, x0);
-            else
-                f4_load(args.x0_prev, (view_base + c + 4) * HW + p0, cnt, VEC, x0);
-            if (recon) Lat4<T>::load(xt_p, (view_base + c + 4) * HW + p0, cnt, VEC, xt);
+            for (int c = 0; c < 4; ++c) {
+                if (c >= cn) break;
+                float x[4], y[4], pr[4];
+                Lat4<T>::unpack(xt[c], x);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) y[i] = recon_one(args.coef, x[i], x0[c][i], pr[i]);
+                const size_t e = view_base + (size_t)(cg + c) * plane;
+                Lat4<T>::store(xn_p, e, cnt, VEC, y);
+                if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, VEC, pr);
+            }
         }
     }
 }
 
-size_t tile_smem_bytes(int K, int a) {
-    return sizeof(geocache_camera) * kTileMaxAnchors + (size_t)K * a * kTile * 9 + 2 * kTile;
+template <typename T, int K, int MODE>
+static cudaError_t launch_quad(const TransportArgs& t, cudaStream_t s) {
+    const int HW = t.H * t.W;
+    const uintptr_t al = (uintptr_t)t.x0_new | (uintptr_t)t.x0_prev | (uintptr_t)t.x0_out | (uintptr_t)t.x_t |
+                         (uintptr_t)t.x_next | (uintptr_t)t.pred_out | (uintptr_t)t.keep | (uintptr_t)t.valid;
+    const bool vec = (HW % 4 == 0) && (al % 16 == 0);
+    const int quads = (HW + 3) / 4;
+    dim3 grid((quads + kThreads - 1) / kThreads, t.N, t.B);
+    if (vec)
+        transport_quad_kernel<T, K, MODE, true><<<grid, kThreads, 0, s>>>(t);
+    else
+        transport_quad_kernel<T, K, MODE, false><<<grid, kThreads, 0, s>>>(t);
+    return cudaGetLastError();
 }
 
 template <typename T, int K>
 static cudaError_t launch_transport_t(const TransportArgs& t, cudaStream_t s) {
-    const int HW = t.H * t.W;
-    if (t.a <= kTileMaxAnchors) {
-        const uintptr_t al = (uintptr_t)t.x0_new | (uintptr_t)t.x0_prev | (uintptr_t)t.x0_out |
-                             (uintptr_t)t.x_t | (uintptr_t)t.x_next | (uintptr_t)t.pred_out;
-        const bool vec = (HW % 4 == 0) && (al % 16 == 0);
-        const size_t smem = tile_smem_bytes(K, t.a);
-        dim3 grid((HW + kTile - 1) / kTile, t.N, t.B);
-        auto kern = vec ? transport_tile_kernel<T, K, true> : transport_tile_kernel<T, K, false>;
-        if (smem > 48 * 1024) {
-            cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-            if (e != cudaSuccess) return e;
-        }
-        kern<<<grid, kTile, smem, s>>>(t);
-        return cudaGetLastError();
+    switch (t.mode) {
+        case GEOCACHE_CORR_MASK: return launch_quad<T, K, GEOCACHE_CORR_MASK>(t, s);
+        case GEOCACHE_CORR_TABLE: return launch_quad<T, K, GEOCACHE_CORR_TABLE>(t, s);
+        default: return launch_quad<T, K, GEOCACHE_CORR_GEOMETRY>(t, s);
     }
-    dim3 grid((HW + 255) / 256, t.N, t.B);
-    TransportArgs c = t;
-    const int chunk = t.C <= 4 ? 4 : 16;
-    for (int c0 = 0; c0 < t.C; c0 += chunk) {
-        c.c0 = c0;
-        c.cn = t.C - c0 < chunk ? t.C - c0 : chunk;
-        if (c.cn <= 4)
-            transport_pixel_kernel<T, K, 4><<<grid, 256, 0, s>>>(c);
-        else
-            transport_pixel_kernel<T, K, 16><<<grid, 256, 0, s>>>(c);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-    }
-    return cudaSuccess;
 }
 
-int transport_launch_count(int a, int C, int in_place) {
-    int n = a <= kTileMaxAnchors ? 1 : (C + (C <= 4 ? 4 : 16) - 1) / (C <= 4 ? 4 : 16);
-    return n + (in_place ? 1 : 0);
-}
+int transport_launch_count(int, int, int in_place) { return 1 + (in_place ? 1 : 0); }
 
 cudaError_t launch_transport(const TransportArgs& t, cudaStream_t s) {
     if (t.lat_dtype == GEOCACHE_BF16)
