@@ -42,7 +42,7 @@ def parse():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="batch128")
     p.add_argument("--assets", type=int, default=64, help="assets per GPU (the batch128 sweep axis)")
-    p.add_argument("--corr", default="mask", choices=["mask", "geometry", "table"])
+    p.add_argument("--corr", default="sparse", choices=["sparse", "mask", "geometry", "table"])
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-assets", type=int, default=4, help="assets in the oracle's timed sample")
@@ -84,7 +84,7 @@ def step_bytes(w):
 class Trajectory:
     """Device state of one batch's trajectory and the loop over its steps."""
 
-    def __init__(self, w, dev, corr_mode="mask"):
+    def __init__(self, w, dev, corr_mode="sparse"):
         import torch
         from paper_2608_13255_gb300 import geocache as gc
         from paper_2608_13255_gb300 import synth
@@ -94,16 +94,24 @@ class Trajectory:
         self.valid = torch.from_numpy(w.valid).to(dev)
         self.cams = torch.from_numpy(w.cams).to(dev)
         self.tau = torch.zeros(w.B, dtype=torch.float32, device=dev)
-        idx = wt = keep = None
+        idx = wt = keep = tile_ptr = records = None
         if corr_mode == "table":
             shp = (w.B, w.N, w.N, w.H, w.W, w.K)
             idx = torch.empty(shp, dtype=torch.int32, device=dev)
             wt = torch.empty(shp, dtype=torch.float32, device=dev)
-        if corr_mode == "mask":
+        if corr_mode in ("mask", "sparse"):
             keep = torch.empty((w.B, w.N, w.N, w.H, w.W), dtype=torch.uint8, device=dev)
-        mode = {"mask": gc.CORR_MASK, "table": gc.CORR_TABLE, "geometry": gc.CORR_GEOMETRY}[corr_mode]
+        if corr_mode == "sparse":
+            tile_ptr = torch.empty(w.B * w.N * w.N * gc.tiles_per_view(w.H, w.W) + 1, dtype=torch.int32, device=dev)
+            c0 = gc.make_corr(self.pos, self.valid, self.cams, self.tau, K=w.K, tol_frac=w.tol_frac, keep=keep,
+                              tile_ptr=tile_ptr, mode=gc.CORR_MASK)
+            records = torch.empty((max(gc.record_count(c0), 1), 4), dtype=torch.int32, device=dev)
+        mode = {"mask": gc.CORR_MASK, "table": gc.CORR_TABLE, "geometry": gc.CORR_GEOMETRY,
+                "sparse": gc.CORR_SPARSE}[corr_mode]
         self.corr = gc.make_corr(self.pos, self.valid, self.cams, self.tau, idx, wt, K=w.K, tol_frac=w.tol_frac,
-                                 mode=mode, keep=keep)
+                                 mode=mode, keep=keep, tile_ptr=tile_ptr, records=records)
+        nws = self.corr.workspace_floats(w.C)
+        self.workspace = torch.empty(max(nws, 4), dtype=torch.float32, device=dev) if nws else None
         xT, x0 = synth.initial_latents(w)
         lat = torch.bfloat16 if w.dtype == "bf16" else torch.float32
         self.x = torch.from_numpy(xT).to(dev).to(lat)
@@ -140,6 +148,8 @@ class Trajectory:
         launches = 0
         gc.build_corr(self.corr)
         launches += 1 + (1 if (self.corr.idx is not None or self.corr.keep is not None) else 0)
+        if self.corr.c.mode == gc.CORR_SPARSE:
+            launches += 3  # tile counts, their scan, the records
         cache = None
         for t in range(w.S):
             anchors, full = gc.rotate_anchors(w.N, w.a, t, w.S, self.sched)
@@ -153,11 +163,11 @@ class Trajectory:
                     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                     e0.record()
                 gc.transport_step(self.corr, anchors, w.C, self.anchor_x0[t], cache, out, self.x, self.x,
-                                  self.recon[t])
+                                  self.recon[t], workspace=self.workspace)
                 if events is not None:
                     e1.record()
                     events.append((e0, e1))
-                launches += gc.transport_launches(w.a, w.C, in_place=False)
+                launches += gc.transport_launches(w.a, w.N, self.corr.c.mode, in_place=False)
                 cache = out
         return launches
 

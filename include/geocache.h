@@ -7,8 +7,9 @@
  * ---------------------------------------
  * - Pointers marked "device" are CUDA device addresses on the current device
  *   (e.g. torch tensors' data_ptr()); pointers marked "host" are ordinary host
- *   memory.  The caller owns every buffer; the library keeps no device state
- *   between calls and allocates no memory.
+ *   memory.  The caller owns every buffer and the library allocates no
+ *   memory; its only device-resident state is a 4-byte status word that
+ *   kernels set when a bounded wait gives up (geocache_device_status).
  * - Every device-side entry point is asynchronous on `stream` (a cudaStream_t,
  *   NULL = the legacy default stream) and returns after enqueueing its kernels.
  * - Latents are NCHW per view with the views on the batch axis:
@@ -30,6 +31,7 @@ extern "C" {
 #define GEOCACHE_ABI_VERSION 1
 #define GEOCACHE_MAX_VIEWS 64   /* N <= 64 */
 #define GEOCACHE_MAX_CHANNELS 1024
+#define GEOCACHE_TILE_TOKENS 1024 /* tokens per tile of the sparse operator (row-major token order) */
 
 typedef enum {
     GEOCACHE_OK = 0,
@@ -37,7 +39,7 @@ typedef enum {
     GEOCACHE_ESHAPE = -2,   /* a size is out of range */
     GEOCACHE_EDTYPE = -3,   /* unsupported latent dtype */
     GEOCACHE_ECUDA = -4,    /* a CUDA call or kernel launch failed */
-    GEOCACHE_ETIMEOUT = -5, /* reserved: a bounded device wait gave up */
+    GEOCACHE_ETIMEOUT = -5, /* a bounded device wait gave up (see geocache_device_status) */
     GEOCACHE_EDEVICE = -6,  /* no usable CUDA device */
     GEOCACHE_EALIAS = -7    /* buffers overlap in a way the call does not allow */
 } geocache_status;
@@ -55,14 +57,26 @@ typedef enum {
     GEOCACHE_PRED_VELOCITY = 3  /* FM: u = (x_sigma - x0) / sigma */
 } geocache_pred;
 
-/* How geocache_transport_step obtains the taps of G_{u->v}.  All three give
- * bit-identical taps and weights. */
+/* How geocache_transport_step obtains the taps of G_{u->v}.  All four give
+ * bit-identical taps, weights and results. */
 typedef enum {
     GEOCACHE_CORR_GEOMETRY = 0, /* recompute every tap test from pos/valid/cams/tau */
     GEOCACHE_CORR_TABLE = 1,    /* read idx/w written by geocache_build_corr (or supplied by the caller) */
-    GEOCACHE_CORR_MASK = 2      /* read the 1-byte keep masks written by geocache_build_corr; recompute
-                                   the projection and weights only where a tap is kept (fastest) */
+    GEOCACHE_CORR_MASK = 2,     /* read the 1-byte keep masks written by geocache_build_corr; recompute
+                                   the projection and weights only where a tap is kept */
+    GEOCACHE_CORR_SPARSE = 3    /* read the sparse tap records written by geocache_build_corr and apply
+                                   them record-parallel into a workspace (fastest) */
 } geocache_corr_mode;
+
+/* One kept (target token, source view) row of G_{u->v} in sparse form: the
+ * bilinear footprint's top-left tap and fractions, from which the kept taps'
+ * indices and renormalised weights follow exactly as in the tables.
+ * 16 bytes. */
+typedef struct {
+    int32_t token_mask;   /* target token p (bits 0..27) | keep mask << 28 (bit k = tap k kept) */
+    int32_t q_tl;         /* source index of the top-left tap (row*W + col; may be -1 or -W-1 off-image) */
+    float fx, fy;         /* footprint fractions (K = 4); 0 for K = 1, where q_tl is the single tap */
+} geocache_tap_record;
 
 /* Pinhole camera, world -> camera: x_c = R x_w + t (R row-major), +z forward,
  * pixel x right, pixel y down, token (i, j) centred at (i + 0.5, j + 0.5).
@@ -94,6 +108,11 @@ typedef struct {
                                        -1 = tap not kept; or NULL (tables not built) */
     float* w;                       /* device [B,N(v),N(u),H,W,K] f32 weights, 0 where idx = -1; or NULL */
     uint8_t* keep;                  /* device [B,N(v),N(u),H,W] u8: bit k set iff tap k is kept; or NULL */
+    int32_t* tile_ptr;              /* device [B*N*N*T + 1] i32 (T = ceil(H*W / GEOCACHE_TILE_TOKENS)):
+                                       records of (b, v, u, tile) are records[tile_ptr[i] .. tile_ptr[i+1]),
+                                       i = ((b*N + v)*N + u)*T + tile; or NULL */
+    geocache_tap_record* records;   /* device [max_records], sorted by (b, v, u, token); or NULL */
+    int64_t max_records;            /* capacity of records */
     geocache_corr_mode mode;        /* taps used by geocache_transport_step */
 } geocache_corr;
 
@@ -140,12 +159,33 @@ typedef struct {
  * Reads corr->pos, corr->valid, corr->cams; writes corr->tau[B] and, for
  * every ordered pair (v, u), the tables idx/w (when both are non-NULL) and
  * the keep masks (when keep is non-NULL): the diagonal u == v and
- * background targets hold idx -1 / w 0 / keep 0.
+ * background targets hold idx -1 / w 0 / keep 0.  When tile_ptr is given
+ * (it needs keep) the tile offsets of the sparse form are written, and when
+ * records is also given the records are written; this last part reads the
+ * record count back to the host (the call then synchronises `stream`) and
+ * fails with ESHAPE if it exceeds max_records (see geocache_corr_record_count).
  * Sizes: 1 <= B, 2 <= N <= GEOCACHE_MAX_VIEWS, 1 <= H, W <= 16384,
- * K in {1, 4}, 0 < tol_frac.  tau must not overlap the other buffers.
- * Returns GEOCACHE_OK, EINVAL (NULL / bad K / tol_frac), ESHAPE, ECUDA.
+ * K in {1, 4}, 0 < tol_frac.  Outputs must not overlap the inputs.
+ * Returns GEOCACHE_OK, EINVAL (NULL / bad K / tol_frac), ESHAPE, EALIAS, ECUDA.
  * ------------------------------------------------------------------------ */
 int geocache_build_corr(geocache_corr* corr, void* stream);
+
+/* --------------------------------------------------------------------------
+ * geocache_corr_record_count -- number of sparse records of a batch (the
+ * kept (target token, source view) rows of every G_{u->v}): builds tau, the
+ * keep masks and tile_ptr (corr->keep and corr->tile_ptr are required), then
+ * synchronises `stream` and returns the count in *count.  Allocate
+ * max_records >= *count records and call geocache_build_corr to fill them.
+ * Returns GEOCACHE_OK, EINVAL, ESHAPE, ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_corr_record_count(geocache_corr* corr, int64_t* count, void* stream);
+
+/* --------------------------------------------------------------------------
+ * geocache_transport_workspace -- number of floats of workspace that
+ * geocache_transport_step needs for `corr` with C channels (0 unless
+ * corr->mode is GEOCACHE_CORR_SPARSE, then max_records * C).  Host only.
+ * ------------------------------------------------------------------------ */
+int64_t geocache_transport_workspace(const geocache_corr* corr, int C);
 
 /* --------------------------------------------------------------------------
  * geocache_transport_step -- one cached sampler step (Eq. 1 and the
@@ -170,14 +210,19 @@ int geocache_build_corr(geocache_corr* corr, void* stream);
  *             view (bf16 stores round to nearest even); x_next may equal x_t.
  *             Ignored when recon is NULL.
  *   C         1 <= C <= GEOCACHE_MAX_CHANNELS.
+ *   workspace device f32 scratch of at least geocache_transport_workspace(corr, C)
+ *             floats (NULL when that is 0); its contents are not preserved
+ *             between calls, and calls sharing a workspace must not overlap.
  * corr must have been filled by geocache_build_corr (tau; idx/w in
- * GEOCACHE_CORR_TABLE mode; keep in GEOCACHE_CORR_MASK mode).
+ * GEOCACHE_CORR_TABLE mode; keep in GEOCACHE_CORR_MASK mode; keep, tile_ptr
+ * and records in GEOCACHE_CORR_SPARSE mode).
  * Returns GEOCACHE_OK, EINVAL, ESHAPE, EDTYPE, EALIAS, ECUDA.
  * ------------------------------------------------------------------------ */
 int geocache_transport_step(const geocache_corr* corr, const int32_t* anchors, int a, int C,
                             const float* x0_anchor_new, const float* x0_prev, float* x0_out,
                             const void* x_t, void* x_next, geocache_dtype lat_dtype,
-                            const geocache_recon* recon, void* stream);
+                            const geocache_recon* recon, float* workspace, int64_t workspace_floats,
+                            void* stream);
 
 /* --------------------------------------------------------------------------
  * geocache_reconstruct -- full-step passthrough (Sec. 3.2: at a full step the
@@ -213,6 +258,16 @@ int geocache_is_full_step(int step, int S, const geocache_schedule* sched);
  * ------------------------------------------------------------------------ */
 int geocache_rotate_anchors(int N, int a, int step, int S, const geocache_schedule* sched,
                             int32_t* anchors_out, int* is_full_out);
+
+/* --------------------------------------------------------------------------
+ * geocache_device_status -- synchronises `stream`, then reads and clears the
+ * device status word.  Every wait inside the kernels (the completion of their
+ * own bulk copies into shared memory) is bounded in time; a CTA whose wait
+ * runs out sets the word and returns without writing its outputs, so the
+ * context stays usable.  Returns GEOCACHE_OK, ETIMEOUT (some call since the
+ * last check left outputs incomplete) or ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_device_status(void* stream);
 
 /* Thread-local description of the last non-OK status of this thread ("" if
  * none).  The pointer stays valid until the thread's next library call. */

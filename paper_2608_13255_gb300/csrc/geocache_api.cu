@@ -87,11 +87,31 @@ int make_coef(const geocache_recon* r, geocache::ReconCoef* c) {
 
 size_t lat_bytes(int dtype) { return dtype == GEOCACHE_BF16 ? 2 : 4; }
 
+// total record count of the sparse form (synchronises the stream)
+int read_total(const geocache_corr* c, int64_t* total, cudaStream_t s) {
+    const size_t n = (size_t)c->B * c->N * c->N * geocache::tiles_per_view(c->H, c->W);
+    int32_t v = 0;
+    cudaError_t e = cudaMemcpyAsync(&v, c->tile_ptr + n, sizeof v, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the record count");
+    if (v < 0) return fail(GEOCACHE_ESHAPE, "the sparse form has more than 2^31-1 records");
+    *total = v;
+    return GEOCACHE_OK;
+}
+
 }  // namespace
 
 extern "C" {
 
 int geocache_abi_version(void) { return GEOCACHE_ABI_VERSION; }
+
+int geocache_device_status(void* stream) {
+    unsigned int word = 0;
+    cudaError_t e = geocache::read_device_error(&word, true, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the device status word");
+    if (word) return fail(GEOCACHE_ETIMEOUT, "a bounded device wait gave up (status word 0x%x); outputs of that call are incomplete", word);
+    return ok();
+}
 
 const char* geocache_last_error(void) { return g_last_error.c_str(); }
 
@@ -120,6 +140,19 @@ int geocache_build_corr(geocache_corr* c, void* stream) {
     if (c->keep && (overlap(c->keep, texels * c->N, c->pos, texels * 12) || overlap(c->keep, texels * c->N, c->valid, texels) ||
                     overlap(c->keep, texels * c->N, c->tau, sizeof(float) * c->B)))
         return fail(GEOCACHE_EALIAS, "keep overlaps an input");
+    if (c->tile_ptr && !c->keep) return fail(GEOCACHE_EINVAL, "tile_ptr needs keep");
+    if (c->records && !c->tile_ptr) return fail(GEOCACHE_EINVAL, "records need tile_ptr");
+    if (c->records && (c->max_records < 0 || ((uintptr_t)c->records & 15)))
+        return fail(GEOCACHE_EINVAL, "records must be 16-byte aligned with max_records >= 0");
+    if (c->tile_ptr) {
+        const size_t nt = (size_t)c->B * c->N * c->N * geocache::tiles_per_view(c->H, c->W) + 1;
+        if (overlap(c->tile_ptr, nt * 4, c->keep, texels * c->N) || overlap(c->tile_ptr, nt * 4, c->pos, texels * 12) ||
+            (c->records && overlap(c->tile_ptr, nt * 4, c->records, (size_t)c->max_records * 16)))
+            return fail(GEOCACHE_EALIAS, "tile_ptr overlaps another buffer");
+    }
+    if (c->records && (overlap(c->records, (size_t)c->max_records * 16, c->pos, texels * 12) ||
+                       overlap(c->records, (size_t)c->max_records * 16, c->keep, texels * c->N)))
+        return fail(GEOCACHE_EALIAS, "records overlap another buffer");
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = geocache::launch_tau(c->pos, c->valid, c->B, c->N, c->H, c->W, c->tol_frac, c->tau, s);
     if (e != cudaSuccess) return cuda_fail(e, "tau kernel launch");
@@ -127,12 +160,44 @@ int geocache_build_corr(geocache_corr* c, void* stream) {
         e = geocache::launch_build_corr(*c, s);
         if (e != cudaSuccess) return cuda_fail(e, "correspondence kernel launch");
     }
+    if (c->tile_ptr) {
+        e = geocache::launch_tile_ptr(*c, s);
+        if (e != cudaSuccess) return cuda_fail(e, "tile-offset kernel launch");
+    }
+    if (c->records) {
+        int64_t total = 0;
+        st = read_total(c, &total, s);
+        if (st) return st;
+        if (total > c->max_records)
+            return fail(GEOCACHE_ESHAPE, "the sparse form has %lld records but max_records is %lld",
+                        (long long)total, (long long)c->max_records);
+        e = geocache::launch_fill_records(*c, s);
+        if (e != cudaSuccess) return cuda_fail(e, "record kernel launch");
+    }
     return ok();
+}
+
+int geocache_corr_record_count(geocache_corr* c, int64_t* count, void* stream) {
+    if (!c || !count) return fail(GEOCACHE_EINVAL, "corr and count are required");
+    if (!c->keep || !c->tile_ptr) return fail(GEOCACHE_EINVAL, "counting records needs keep and tile_ptr");
+    geocache_corr d = *c;
+    d.records = nullptr;
+    d.idx = nullptr;
+    d.w = nullptr;
+    int st = geocache_build_corr(&d, stream);
+    if (st) return st;
+    return read_total(c, count, (cudaStream_t)stream);
+}
+
+int64_t geocache_transport_workspace(const geocache_corr* c, int C) {
+    if (!c || C < 1 || c->mode != GEOCACHE_CORR_SPARSE || c->max_records < 0) return 0;
+    return c->max_records * (int64_t)C;
 }
 
 int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int a, int C,
                             const float* x0_anchor_new, const float* x0_prev, float* x0_out, const void* x_t,
-                            void* x_next, geocache_dtype lat_dtype, const geocache_recon* recon, void* stream) {
+                            void* x_next, geocache_dtype lat_dtype, const geocache_recon* recon, float* workspace,
+                            int64_t workspace_floats, void* stream) {
     if (!c) return fail(GEOCACHE_EINVAL, "corr is NULL");
     int st = check_sizes(c->B, c->N, c->H, c->W);
     if (st) return st;
@@ -146,6 +211,13 @@ int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int 
     } else if (c->mode == GEOCACHE_CORR_MASK) {
         if (!c->keep || !c->pos || !c->valid || !c->cams || !c->tau)
             return fail(GEOCACHE_EINVAL, "mask mode needs keep, pos, valid, cams and tau");
+    } else if (c->mode == GEOCACHE_CORR_SPARSE) {
+        if (!c->tile_ptr || !c->records || ((uintptr_t)c->records & 15))
+            return fail(GEOCACHE_EINVAL, "sparse mode needs tile_ptr and 16-byte aligned records");
+        if (a < c->N && (!workspace || workspace_floats < c->max_records * (int64_t)C))
+            return fail(GEOCACHE_EINVAL, "sparse mode needs a workspace of max_records * C = %lld floats",
+                        (long long)(c->max_records * (int64_t)C));
+        if (((uintptr_t)workspace & 15)) return fail(GEOCACHE_EINVAL, "workspace must be 16-byte aligned");
     } else {
         return fail(GEOCACHE_EINVAL, "unknown corr mode %d", (int)c->mode);
     }
@@ -179,13 +251,25 @@ int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int 
              overlap(recon->pred_out, n_all * 4, x0_prev, n_all * 4) || overlap(recon->pred_out, n_all * 4, x_t, n_all * lb)))
             return fail(GEOCACHE_EALIAS, "pred_out overlaps another buffer");
     }
+    if (c->mode == GEOCACHE_CORR_SPARSE && workspace) {
+        const size_t wb = (size_t)workspace_floats * 4, lb = lat_bytes(lat_dtype);
+        if (overlap(workspace, wb, x0_out, n_all * 4) || overlap(workspace, wb, x0_prev, n_all * 4) ||
+            overlap(workspace, wb, x0_anchor_new, n_anc * 4) ||
+            (recon && (overlap(workspace, wb, x_next, n_all * lb) || overlap(workspace, wb, x_t, n_all * lb))))
+            return fail(GEOCACHE_EALIAS, "workspace overlaps another buffer");
+    }
     geocache::TransportArgs t{};
     t.B = c->B; t.N = c->N; t.H = c->H; t.W = c->W; t.C = C; t.K = c->K; t.a = a;
     t.mode = c->mode;
-    t.write_anchor_rows = (x0_out != x0_prev);
+    // the sparse mode gathers in a kernel that completes before any row is
+    // written, so an in-place update needs no separate anchor-row pass
+    t.write_anchor_rows = (x0_out != x0_prev) || c->mode == GEOCACHE_CORR_SPARSE;
     t.lat_dtype = lat_dtype;
     t.pos = c->pos; t.valid = c->valid; t.cams = c->cams; t.tau = c->tau; t.idx = c->idx; t.w = c->w;
     t.keep = c->keep;
+    t.tile_ptr = c->tile_ptr;
+    t.records = c->records;
+    t.workspace = workspace;
     t.x0_new = x0_anchor_new; t.x0_prev = x0_prev; t.x0_out = x0_out;
     t.x_t = x_t; t.x_next = x_next; t.pred_out = recon ? recon->pred_out : nullptr;
     t.coef = coef;

@@ -139,6 +139,22 @@ __device__ __forceinline__ void taps_from_mask(const Footprint& f, int mask, int
         if (t.q[k] >= 0) t.w[k] = __fmul_rn(raw[k], rs);
 }
 
+// The same indices and weights from a sparse record (top-left tap q_tl and the
+// footprint fractions fx, fy stored by the build): ax = (1-fx, fx),
+// ay = (1-fy, fy) are recomputed exactly as footprint() forms them.
+template <int K>
+__device__ __forceinline__ void taps_from_record(int mask, int q_tl, float fx, float fy, int W, Taps& t) {
+    Footprint f;
+    f.ax[0] = __fsub_rn(1.0f, fx);
+    f.ax[1] = fx;
+    f.ay[0] = __fsub_rn(1.0f, fy);
+    f.ay[1] = fy;
+    // i0 + j0*W = q_tl; taps_from_mask only uses (j0 + dj)*W + (i0 + di)
+    f.i0 = q_tl;
+    f.j0 = 0;
+    taps_from_mask<K>(f, mask, W, t);
+}
+
 // Taps of target point X in source view u (pos_u [H*W*3], valid_u [H*W]):
 // footprint, per-tap tests, renormalised weights.  *mask_out (optional)
 // receives the keep mask.

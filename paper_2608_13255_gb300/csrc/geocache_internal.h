@@ -32,6 +32,9 @@ struct TransportArgs {
     const int32_t* idx;
     const float* w;
     const uint8_t* keep;
+    const int32_t* tile_ptr;
+    const geocache_tap_record* records;
+    float* workspace;
     const float* x0_new;
     const float* x0_prev;
     float* x0_out;
@@ -46,10 +49,17 @@ struct TransportArgs {
 cudaError_t launch_tau(const float* pos, const uint8_t* valid, int B, int N, int H, int W,
                        float tol_frac, float* tau, cudaStream_t s);
 cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s);
+// sparse form: per-tile record counts and their exclusive prefix sum in
+// tile_ptr (tile_ptr[n] = total, or -1 when the total exceeds INT32_MAX)
+cudaError_t launch_tile_ptr(const geocache_corr& c, cudaStream_t s);
+cudaError_t launch_fill_records(const geocache_corr& c, cudaStream_t s);
+int tiles_per_view(int H, int W);
 cudaError_t launch_transport(const TransportArgs& t, cudaStream_t s);
 int transport_launch_count(int a, int C, int in_place);
 cudaError_t launch_copy_anchor_rows(const TransportArgs& t, cudaStream_t s);
 cudaError_t launch_reconstruct(const void* x_t, const float* x0, void* x_next, int lat_dtype, int64_t n,
                                const ReconCoef& coef, float* pred_out, float* x0_store, cudaStream_t s);
+
+cudaError_t read_device_error(unsigned int* out, bool clear, cudaStream_t s);
 
 }  // namespace geocache

@@ -165,6 +165,167 @@ cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+// ---------------------------------------------------- sparse operator --
+// G_{u->v} in tile-CSR form: for each (asset b, target view v, source view u,
+// tile of GEOCACHE_TILE_TOKENS tokens) the records of its kept rows, in token
+// order; tile_ptr holds the exclusive prefix sum of the per-tile counts.
+int tiles_per_view(int H, int W) { return (H * W + GEOCACHE_TILE_TOKENS - 1) / GEOCACHE_TILE_TOKENS; }
+__device__ __forceinline__ int tiles_per_view_dev(int H, int W) {
+    return (H * W + GEOCACHE_TILE_TOKENS - 1) / GEOCACHE_TILE_TOKENS;
+}
+
+// count of kept rows (non-zero keep bytes) of each (b, v, u, tile)
+__global__ void __launch_bounds__(256) tile_count_kernel(const uint8_t* __restrict__ keep, int N, int HW, int T,
+                                                         int32_t* __restrict__ cnt) {
+    const int tile = blockIdx.x, vu = blockIdx.y, b = blockIdx.z;
+    const uint8_t* row = keep + ((size_t)b * N * N + vu) * HW;
+    const int tile0 = tile * GEOCACHE_TILE_TOKENS;
+    int c = 0;
+    for (int i = threadIdx.x; i < GEOCACHE_TILE_TOKENS; i += blockDim.x) {
+        const int p = tile0 + i;
+        if (p < HW && __ldg(row + p)) ++c;
+    }
+    c = __reduce_add_sync(0xffffffffu, c);
+    __shared__ int s[8];
+    if ((threadIdx.x & 31) == 0) s[threadIdx.x >> 5] = c;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int tot = 0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += s[w];
+        cnt[((size_t)b * N * N + vu) * T + tile] = tot;
+    }
+}
+
+// in-place exclusive prefix sum of n counts by one CTA; a[n] = total, or -1
+// when the total does not fit an int32
+__global__ void __launch_bounds__(1024) exclusive_scan_kernel(int32_t* a, long long n) {
+    __shared__ long long s_warp[32];
+    __shared__ long long s_carry;
+    constexpr int kItems = 8;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    if (t == 0) s_carry = 0;
+    __syncthreads();
+    for (long long base = 0; base < n; base += 1024LL * kItems) {
+        long long v[kItems];
+        long long sum = 0;
+#pragma unroll
+        for (int i = 0; i < kItems; ++i) {
+            const long long idx = base + (long long)t * kItems + i;
+            v[i] = idx < n ? a[idx] : 0;
+            sum += v[i];
+        }
+        long long incl = sum;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const long long y = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += y;
+        }
+        if (lane == 31) s_warp[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            long long w = s_warp[lane];
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const long long y = __shfl_up_sync(0xffffffffu, w, off);
+                if (lane >= off) w += y;
+            }
+            s_warp[lane] = w;
+        }
+        __syncthreads();
+        long long run = s_carry + (warp ? s_warp[warp - 1] : 0) + incl - sum;
+#pragma unroll
+        for (int i = 0; i < kItems; ++i) {
+            const long long idx = base + (long long)t * kItems + i;
+            if (idx < n) a[idx] = run > 0x7fffffffLL ? -1 : (int32_t)run;
+            run += v[i];
+        }
+        __syncthreads();
+        if (t == 0) s_carry += s_warp[31];
+        __syncthreads();
+    }
+    if (t == 0) a[n] = s_carry > 0x7fffffffLL ? -1 : (int32_t)s_carry;
+}
+
+cudaError_t launch_tile_ptr(const geocache_corr& c, cudaStream_t s) {
+    const int HW = c.H * c.W, T = tiles_per_view(c.H, c.W);
+    dim3 grid(T, c.N * c.N, c.B);
+    tile_count_kernel<<<grid, 256, 0, s>>>(c.keep, c.N, HW, T, c.tile_ptr);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    exclusive_scan_kernel<<<1, 1024, 0, s>>>(c.tile_ptr, (long long)c.B * c.N * c.N * T);
+    return cudaGetLastError();
+}
+
+// records of one (b, v, u, tile): kept rows in token order, each with its
+// footprint's top-left tap and fractions (recomputed with the same device
+// functions as the tables, so the taps and weights they give are identical)
+template <int K>
+__global__ void __launch_bounds__(256) fill_records_kernel(const float* __restrict__ pos,
+                                                           const geocache_camera* __restrict__ cams,
+                                                           const uint8_t* __restrict__ keep,
+                                                           const int32_t* __restrict__ tile_ptr, int N, int H,
+                                                           int W, int T, geocache_tap_record* __restrict__ rec,
+                                                           long long max_records) {
+    const int tile = blockIdx.x, vu = blockIdx.y, b = blockIdx.z;
+    const int v = vu / N, u = vu % N;
+    const int HW = H * W;
+    const int t = threadIdx.x;
+    __shared__ geocache_camera s_cam;
+    __shared__ int s_warp[8];
+    if (t < 16) reinterpret_cast<float*>(&s_cam)[t] = __ldg(reinterpret_cast<const float*>(cams + (size_t)b * N + u) + t);
+    const int tile0 = tile * GEOCACHE_TILE_TOKENS;
+    const uint8_t* row = keep + ((size_t)b * N * N + vu) * HW;
+    uint32_t m[4];
+    int mine = 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int p = tile0 + 4 * t + i;
+        m[i] = p < HW ? __ldg(row + p) : 0u;
+        mine += m[i] != 0;
+    }
+    // exclusive scan over the CTA (token order)
+    const int lane = t & 31, warp = t >> 5;
+    int incl = mine;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    int base = 0;
+    for (int w = 0; w < warp; ++w) base += s_warp[w];
+    long long r = (long long)__ldg(tile_ptr + ((size_t)b * N * N + vu) * T + tile) + base + incl - mine;
+    const size_t tv0 = ((size_t)b * N + v) * HW;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        if (!m[i]) continue;
+        const int p = tile0 + 4 * t + i;
+        Footprint f;
+        footprint<K>(s_cam, __ldg(pos + 3 * (tv0 + p)), __ldg(pos + 3 * (tv0 + p) + 1), __ldg(pos + 3 * (tv0 + p) + 2),
+                     H, W, f);
+        geocache_tap_record out;
+        out.token_mask = p | (int)(m[i] << 28);
+        out.q_tl = f.j0 * W + f.i0;
+        out.fx = K == 4 ? f.ax[1] : 0.0f;
+        out.fy = K == 4 ? f.ay[1] : 0.0f;
+        if (r < max_records) reinterpret_cast<int4*>(rec)[r] = *reinterpret_cast<const int4*>(&out);
+        ++r;
+    }
+}
+
+cudaError_t launch_fill_records(const geocache_corr& c, cudaStream_t s) {
+    const int T = tiles_per_view(c.H, c.W);
+    dim3 grid(T, c.N * c.N, c.B);
+    if (c.K == 4)
+        fill_records_kernel<4><<<grid, 256, 0, s>>>(c.pos, c.cams, c.keep, c.tile_ptr, c.N, c.H, c.W, T, c.records,
+                                                    c.max_records);
+    else
+        fill_records_kernel<1><<<grid, 256, 0, s>>>(c.pos, c.cams, c.keep, c.tile_ptr, c.N, c.H, c.W, T, c.records,
+                                                    c.max_records);
+    return cudaGetLastError();
+}
+
 // ------------------------------------------------- fused transport step --
 // One thread per quad of 4 consecutive tokens of one view (asset b, view v),
 // all channels in groups of 4.  For each group the thread issues 16-byte
@@ -280,145 +441,690 @@ __device__ __forceinline__ uint32_t quad_masks(const uint8_t* row, int cnt, bool
     return m;
 }
 
-template <typename T, int K, int MODE, bool VEC>
-__global__ void __launch_bounds__(kThreads) transport_quad_kernel(const TransportArgs args) {
-    const int HW = args.H * args.W;
-    const int p0 = 4 * (blockIdx.x * kThreads + threadIdx.x);
-    if (p0 >= HW) return;
-    const int cnt = HW - p0 < 4 ? HW - p0 : 4;
-    const int v = blockIdx.y, b = blockIdx.z;
+// Fused cached step: a persistent kernel whose CTAs loop over work units
+// (asset b, view v, tile of kTileTokens tokens, group of 4 channels).
+//  * Streaming: one thread arms the unit's mbarrier and issues TMA bulk
+//    copies (cp.async.bulk) of the unit's rows of x0 (the anchor's fresh x0,
+//    or x0(t-1)) and of x_t into a two-stage shared-memory ring, one unit
+//    ahead, so the next unit's rows are in flight while the current unit's
+//    increments are formed.
+//  * Increments (views outside the anchor set): the (token, anchor) pairs
+//    with a kept tap are compacted into a work list (block prefix sum, token
+//    order) and processed one per thread, so the dependent loads of many
+//    tokens overlap:  keep masks -> target position -> projection and
+//    weights -> gathers of the anchor increments x0_new - x0(t-1) at the kept
+//    taps.  Per-anchor sums are combined in anchor order (Eq. 1 with the
+//    multi-anchor aggregation of Sec. 3.2: the mean over covering anchors; a
+//    token without a kept tap keeps x0(t-1)).
+//  * Every token is stored (x0(t)) and reconstructed (x_{t-1}) from the
+//    staged rows with 16-byte stores.
+constexpr int kTileTokens = 4 * kThreads;
+static_assert(kTileTokens == GEOCACHE_TILE_TOKENS, "tile of the sparse form");
+constexpr int kChunk = 4;                        // anchors per work-list round
+constexpr int kPairCap = kChunk * kTileTokens;   // (token, anchor) work items of one round
+constexpr int kStages = 2;
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // bounded mbarrier wait: 2 s
+
+// Device error word (the library's only device-resident state): bit 0 is set
+// when a bounded wait gave up.  Read and cleared by geocache_device_status().
+__device__ unsigned int g_device_error = 0;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(dst)),
+                 "l"(src), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ unsigned long long globaltimer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+// Wait for the phase with the given parity; false after kWaitLimitNs.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer();
+    while (!mbar_try_wait(bar, parity))
+        if (globaltimer() - t0 > kWaitLimitNs) return false;
+    return true;
+}
+
+// exclusive prefix sum over the CTA (deterministic); returns the total
+__device__ __forceinline__ int block_exclusive_scan(int x, int& total, int* s_warp) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int incl = x;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        int w = lane < kThreads / 32 ? s_warp[lane] : 0;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, w, off);
+            if (lane >= off) w += y;
+        }
+        if (lane < kThreads / 32) s_warp[lane] = w;  // inclusive warp totals
+    }
+    __syncthreads();
+    total = s_warp[kThreads / 32 - 1];
+    const int base = warp ? s_warp[warp - 1] : 0;
+    return base + incl - x;
+}
+
+struct FusedShared {
+    float acc[kTileTokens][4];        // per token: sum over covering anchors (anchor order), channel group
+    uint32_t pair[kPairCap];          // work items: token | anchor << 10 | keep mask << 16
+    uint8_t n[kTileTokens];           // per token: number of covering anchors
+    geocache_camera cam[kChunk];
+    int warp[kThreads / 32];
+    uint64_t bar[kStages];
+};
+
+// Taps of work item (token p of view v, anchor slot s2) in the given mode.
+template <int K, int MODE>
+__device__ __forceinline__ void item_taps(const TransportArgs& args, const geocache_camera& cam, int b, int v,
+                                          int s2, int p, int m, size_t tv0, size_t plane, float tau2, Taps& tp) {
+    const int N = args.N;
+    const int u = args.anchors[s2];
+    if (MODE == GEOCACHE_CORR_TABLE) {
+        const size_t row = (((size_t)b * N + v) * N + u) * plane + p;
+        tp.kept = 0;
+#pragma unroll
+        for (int kk = 0; kk < K; ++kk) {
+            tp.q[kk] = __ldg(args.idx + row * K + kk);
+            tp.w[kk] = __ldg(args.w + row * K + kk);
+            tp.kept += tp.q[kk] >= 0;
+        }
+        return;
+    }
+    const float X0 = __ldg(args.pos + 3 * (tv0 + p));
+    const float X1 = __ldg(args.pos + 3 * (tv0 + p) + 1);
+    const float X2 = __ldg(args.pos + 3 * (tv0 + p) + 2);
+    if (MODE == GEOCACHE_CORR_MASK) {
+        Footprint f;
+        footprint<K>(cam, X0, X1, X2, args.H, args.W, f);
+        taps_from_mask<K>(f, m, args.W, tp);
+    } else {
+        const size_t su = ((size_t)b * N + u) * plane;
+        compute_taps<K>(cam, args.pos + 3 * su, args.valid + su, args.H, args.W, X0, X1, X2, tau2, tp);
+    }
+}
+
+// Tap-weighted increment of one anchor at one token, channels [cg, cg+cn).
+template <int K>
+__device__ __forceinline__ void item_increment(const TransportArgs& args, const Taps& tp, int b, int s2, int cg,
+                                               int cn, size_t plane, float (&g)[4]) {
     const int N = args.N, C = args.C, a = args.a;
-    const int slot = args.slot_of[v];
+    const float* xn = args.x0_new + (((size_t)b * a + s2) * C + cg) * plane;
+    const float* xp = args.x0_prev + (((size_t)b * N + args.anchors[s2]) * C + cg) * plane;
+    float dn[K][4], dp[K][4];
+#pragma unroll
+    for (int kk = 0; kk < K; ++kk)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            dn[kk][c] = 0.0f;
+            dp[kk][c] = 0.0f;
+            if (tp.q[kk] >= 0 && c < cn) {
+                const size_t e = (size_t)c * plane + tp.q[kk];
+                dn[kk][c] = __ldg(xn + e);
+                dp[kk][c] = __ldg(xp + e);
+            }
+        }
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        float acc = 0.0f;
+#pragma unroll
+        for (int kk = 0; kk < K; ++kk)
+            if (tp.q[kk] >= 0) acc = __fmaf_rn(tp.w[kk], __fsub_rn(dn[kk][c], dp[kk][c]), acc);
+        g[c] = acc;
+    }
+}
+
+struct UnitCoord {
+    int b, v, tile, cg;
+};
+
+__device__ __forceinline__ UnitCoord unit_coord(long long u, int n_tiles, int n_cg, int N) {
+    UnitCoord c;
+    c.cg = (int)(u % n_cg) * 4;
+    u /= n_cg;
+    c.tile = (int)(u % n_tiles);
+    u /= n_tiles;
+    c.v = (int)(u % N);
+    c.b = (int)(u / N);
+    return c;
+}
+
+// Increments of the tile's covered tokens (views outside the anchor set),
+// left in sh.acc / sh.n for the tile's tokens.
+template <int K, int MODE, bool VEC>
+__device__ __forceinline__ void tile_increments(const TransportArgs& args, FusedShared& sh, int b, int v, int tile0,
+                                                int cg, int cn) {
+    const int HW = args.H * args.W;
+    const int t = threadIdx.x;
+    const int p0 = tile0 + 4 * t;
+    const int cnt = p0 < HW ? (HW - p0 < 4 ? HW - p0 : 4) : 0;
+    const int N = args.N, a = args.a;
     const size_t plane = (size_t)HW;
-    const size_t view_base = ((size_t)b * N + v) * C * plane + p0;   // element (b, v, 0, p0)
+    const size_t tv0 = ((size_t)b * N + v) * plane;
+    float tau2 = 0.0f;
+    if (MODE == GEOCACHE_CORR_GEOMETRY) {
+        const float tu = __ldg(args.tau + b);
+        tau2 = __fmul_rn(tu, tu);
+    }
+    uint32_t fg = 0;
+    if (cnt > 0 && MODE == GEOCACHE_CORR_GEOMETRY) fg = quad_masks(args.valid + tv0 + p0, cnt, VEC);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        *reinterpret_cast<float4*>(sh.acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
+        sh.n[4 * t + i] = 0;
+    }
+    for (int ac = 0; ac < a; ac += kChunk) {
+        const int na = a - ac < kChunk ? a - ac : kChunk;
+        if (MODE != GEOCACHE_CORR_TABLE)
+            for (int i = t; i < na * 16; i += kThreads)
+                reinterpret_cast<float*>(sh.cam)[i] = __ldg(
+                    reinterpret_cast<const float*>(args.cams + (size_t)b * N + args.anchors[ac + (i >> 4)]) + (i & 15));
+        // (token, anchor) work items of this anchor chunk
+        uint32_t m4[4] = {0, 0, 0, 0};  // per own token: 4 bits per anchor of the chunk
+        if (cnt > 0) {
+            if (MODE == GEOCACHE_CORR_MASK) {
+                const uint8_t* krow = args.keep + ((size_t)b * N + v) * N * plane + p0;
+                uint32_t q[kChunk];
+#pragma unroll
+                for (int s2 = 0; s2 < kChunk; ++s2)  // the chunk's masks in flight together
+                    q[s2] = s2 < na ? quad_masks(krow + (size_t)args.anchors[ac + s2] * plane, cnt, VEC) : 0u;
+#pragma unroll
+                for (int s2 = 0; s2 < kChunk; ++s2)
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) m4[i] |= ((q[s2] >> (8 * i)) & 15u) << (4 * s2);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const bool cand = MODE == GEOCACHE_CORR_GEOMETRY ? ((fg >> (8 * i)) & 0xffu) != 0 : i < cnt;
+                    if (cand) m4[i] = (1u << (4 * na)) - 1u;  // every anchor is a candidate
+                }
+            }
+        }
+        int mine = 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int s2 = 0; s2 < kChunk; ++s2) mine += (m4[i] >> (4 * s2)) & 15u ? 1 : 0;
+        int n_items;
+        int k = block_exclusive_scan(mine, n_items, sh.warp);  // barriers inside
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+            for (int s2 = 0; s2 < kChunk; ++s2) {
+                const uint32_t m = (m4[i] >> (4 * s2)) & 15u;
+                if (m) sh.pair[k++] = (uint32_t)(4 * t + i) | ((uint32_t)s2 << 10) | (m << 16);
+            }
+        __syncthreads();
+        for (int r0 = 0; r0 < n_items; r0 += kThreads) {
+            const int j = r0 + t;
+            float g[4] = {0.f, 0.f, 0.f, 0.f};
+            int s_mine = -1, lp = 0;
+            if (j < n_items) {
+                const uint32_t it = sh.pair[j];
+                lp = (int)(it & 1023u);
+                const int s_loc = (int)((it >> 10) & 63u);
+                const int m = (int)((it >> 16) & 15u);
+                Taps tp;
+                item_taps<K, MODE>(args, sh.cam[s_loc], b, v, ac + s_loc, tile0 + lp, m, tv0, plane, tau2, tp);
+                if (tp.kept) {
+                    item_increment<K>(args, tp, b, ac + s_loc, cg, cn, plane, g);
+                    s_mine = s_loc;
+                }
+            }
+            // combine in anchor order (deterministic): anchor s_loc adds in pass s_loc
+            for (int s2 = 0; s2 < na; ++s2) {
+                if (s_mine == s2) {
+                    float4* dst = reinterpret_cast<float4*>(sh.acc[lp]);
+                    float4 cur = *dst;
+                    cur.x = __fadd_rn(cur.x, g[0]);
+                    cur.y = __fadd_rn(cur.y, g[1]);
+                    cur.z = __fadd_rn(cur.z, g[2]);
+                    cur.w = __fadd_rn(cur.w, g[3]);
+                    *dst = cur;
+                    sh.n[lp] += 1;
+                }
+                __syncthreads();
+            }
+        }
+    }
+}
+
+template <typename T, int K, int MODE>
+__global__ void __launch_bounds__(kThreads) transport_fused_kernel(const TransportArgs args, int n_tiles, int n_cg,
+                                                                   long long n_units) {
+    __shared__ FusedShared sh;
+    extern __shared__ __align__(128) unsigned char dyn[];  // [stage]: x0 rows [4][tile] f32, x_t rows [4][tile] T
+    constexpr size_t kStageBytes = 4 * kTileTokens * (sizeof(float) + sizeof(T));
+    const int t = threadIdx.x;
+    const int HW = args.H * args.W;
+    const int N = args.N, C = args.C, a = args.a;
+    const size_t plane = (size_t)HW;
     const bool recon = args.coef.enabled;
     const T* xt_p = static_cast<const T*>(args.x_t);
     T* xn_p = static_cast<T*>(args.x_next);
-    const size_t tv = ((size_t)b * N + v) * plane + p0;              // token p0 of (b, v)
 
-    // which of the quad's tokens have any kept tap (any anchor)
-    uint32_t any_cover = 0;
-    float tau2 = 0.0f;
-    if (slot < 0) {
-        if (MODE == GEOCACHE_CORR_MASK) {
-            const uint8_t* krow = args.keep + ((size_t)b * N + v) * N * plane + p0;
-            for (int s = 0; s < a; ++s) any_cover |= quad_masks(krow + (size_t)args.anchors[s] * plane, cnt, VEC);
-        } else if (MODE == GEOCACHE_CORR_GEOMETRY) {
-            any_cover = quad_masks(args.valid + tv, cnt, VEC);
-            const float tu = __ldg(args.tau + b);
-            tau2 = __fmul_rn(tu, tu);
-        } else {
-            any_cover = 0x01010101u;  // tables: every token is looked up
+    // issue the bulk copies of unit u into stage st (thread 0)
+    auto issue = [&](long long u, int st) {
+        const UnitCoord c = unit_coord(u, n_tiles, n_cg, N);
+        const int tile0 = c.tile * kTileTokens;
+        const int tile_n = HW - tile0 < kTileTokens ? HW - tile0 : kTileTokens;
+        const int cn = C - c.cg < 4 ? C - c.cg : 4;
+        const int slot = args.slot_of[c.v];
+        const float* src = slot >= 0 ? args.x0_new + ((size_t)c.b * a + slot) * C * plane
+                                     : args.x0_prev + ((size_t)c.b * N + c.v) * C * plane;
+        float* s_x0 = reinterpret_cast<float*>(dyn + st * kStageBytes);
+        T* s_xt = reinterpret_cast<T*>(dyn + st * kStageBytes + 4 * kTileTokens * sizeof(float));
+        const uint32_t rx = (uint32_t)tile_n * sizeof(float), rt = (uint32_t)tile_n * sizeof(T);
+        mbar_arrive_expect_tx(&sh.bar[st], cn * (rx + (recon ? rt : 0)));
+        for (int cc = 0; cc < cn; ++cc) {
+            bulk_g2s(s_x0 + cc * kTileTokens, src + (size_t)(c.cg + cc) * plane + tile0, rx, &sh.bar[st]);
+            if (recon)
+                bulk_g2s(s_xt + cc * kTileTokens, xt_p + (((size_t)c.b * N + c.v) * C + c.cg + cc) * plane + tile0, rt,
+                         &sh.bar[st]);
+        }
+    };
+
+    if (t == 0) {
+        for (int st = 0; st < kStages; ++st) mbar_init(&sh.bar[st], 1);
+        fence_mbar_init();
+        if ((long long)blockIdx.x < n_units) issue(blockIdx.x, 0);
+    }
+    __syncthreads();
+    uint32_t parity[kStages] = {0, 0};
+    int st = 0;
+    for (long long u = blockIdx.x; u < n_units; u += gridDim.x) {
+        const long long un = u + gridDim.x;
+        if (t == 0 && un < n_units) {
+            fence_proxy_async();  // the previous unit's shared-memory reads of this stage come first
+            issue(un, st ^ 1);
+        }
+        const UnitCoord c = unit_coord(u, n_tiles, n_cg, N);
+        const int tile0 = c.tile * kTileTokens;
+        const int p0 = tile0 + 4 * t;
+        const int cnt = p0 < HW ? (HW - p0 < 4 ? HW - p0 : 4) : 0;
+        const int cn = C - c.cg < 4 ? C - c.cg : 4;
+        const int slot = args.slot_of[c.v];
+        if (slot < 0) tile_increments<K, MODE, true>(args, sh, c.b, c.v, tile0, c.cg, cn);
+
+        const bool ok = mbar_wait_bounded(&sh.bar[st], parity[st]);
+        if (__syncthreads_or(!ok)) {  // the whole CTA gives up together
+            if (t == 0) atomicOr(&g_device_error, 1u);
+            for (int s2 = 0; s2 < kStages; ++s2) mbar_wait_bounded(&sh.bar[s2], parity[s2]);  // copies in flight
+            return;
+        }
+        parity[st] ^= 1u;
+        if (cnt > 0) {
+            const float* s_x0 = reinterpret_cast<const float*>(dyn + st * kStageBytes);
+            const T* s_xt = reinterpret_cast<const T*>(dyn + st * kStageBytes + 4 * kTileTokens * sizeof(float));
+            const size_t view_base = ((size_t)c.b * N + c.v) * C * plane + p0;
+            float x0[4][4];
+            typename Lat4<T>::Raw xt[4];
+#pragma unroll
+            for (int cc = 0; cc < 4; ++cc) {
+                if (cc >= cn) break;
+                const float4 q = *reinterpret_cast<const float4*>(s_x0 + cc * kTileTokens + 4 * t);
+                x0[cc][0] = q.x; x0[cc][1] = q.y; x0[cc][2] = q.z; x0[cc][3] = q.w;
+                if (recon) xt[cc] = *reinterpret_cast<const typename Lat4<T>::Raw*>(s_xt + cc * kTileTokens + 4 * t);
+            }
+            if (slot < 0) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int n = sh.n[4 * t + i];
+                    if (!n) continue;
+                    const float4 g = *reinterpret_cast<const float4*>(sh.acc[4 * t + i]);
+                    const float gg[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc)
+                        x0[cc][i] = __fadd_rn(x0[cc][i], n == 1 ? gg[cc] : __fdiv_rn(gg[cc], (float)n));
+                }
+            }
+            if (slot < 0 || args.write_anchor_rows) {
+#pragma unroll
+                for (int cc = 0; cc < 4; ++cc) {
+                    if (cc >= cn) break;
+                    Lat4<float>::store(args.x0_out, view_base + (size_t)(c.cg + cc) * plane, cnt, true, x0[cc]);
+                }
+            }
+            if (recon) {
+#pragma unroll
+                for (int cc = 0; cc < 4; ++cc) {
+                    if (cc >= cn) break;
+                    float x[4], y[4], pr[4];
+                    Lat4<T>::unpack(xt[cc], x);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) y[i] = recon_one(args.coef, x[i], x0[cc][i], pr[i]);
+                    const size_t e = view_base + (size_t)(c.cg + cc) * plane;
+                    Lat4<T>::store(xn_p, e, cnt, true, y);
+                    if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, true, pr);
+                }
+            }
+        }
+        __syncthreads();  // stage st and the sums are reused by later units
+        st ^= 1;
+    }
+}
+
+// General path (sizes the bulk copies cannot serve: H*W not a multiple of 8
+// or buffers not 16-byte aligned): one CTA per unit, registers instead of
+// the shared-memory ring.
+template <typename T, int K, int MODE, bool VEC>
+__global__ void __launch_bounds__(kThreads) transport_simple_kernel(const TransportArgs args, int n_tiles, int n_cg) {
+    __shared__ FusedShared sh;
+    const int t = threadIdx.x;
+    const int HW = args.H * args.W;
+    const int N = args.N, C = args.C, a = args.a;
+    const size_t plane = (size_t)HW;
+    const bool recon = args.coef.enabled;
+    const T* xt_p = static_cast<const T*>(args.x_t);
+    T* xn_p = static_cast<T*>(args.x_next);
+    const UnitCoord c = unit_coord(blockIdx.x, n_tiles, n_cg, N);
+    const int tile0 = c.tile * kTileTokens;
+    const int p0 = tile0 + 4 * t;
+    const int cnt = p0 < HW ? (HW - p0 < 4 ? HW - p0 : 4) : 0;
+    const int cn = C - c.cg < 4 ? C - c.cg : 4;
+    const int slot = args.slot_of[c.v];
+    const size_t view_base = ((size_t)c.b * N + c.v) * C * plane + p0;
+    const float* src = slot >= 0 ? args.x0_new + ((size_t)c.b * a + slot) * C * plane + p0
+                                 : args.x0_prev + ((size_t)c.b * N + c.v) * C * plane + p0;
+    float x0[4][4];
+    typename Lat4<T>::Raw xt[4];
+    if (cnt > 0) {
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+            if (cc >= cn) break;
+            if (slot >= 0)
+                f4_load_keep(src, (size_t)(c.cg + cc) * plane, cnt, VEC, x0[cc]);
+            else
+                Lat4<float>::load(src, (size_t)(c.cg + cc) * plane, cnt, VEC, x0[cc]);
+            if (recon) xt[cc] = Lat4<T>::load_raw(xt_p, view_base + (size_t)(c.cg + cc) * plane, cnt, VEC);
         }
     }
+    if (slot < 0) tile_increments<K, MODE, VEC>(args, sh, c.b, c.v, tile0, c.cg, cn);
+    if (cnt <= 0) return;
+    if (slot < 0) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int n = sh.n[4 * t + i];
+            if (!n) continue;
+            const float4 g = *reinterpret_cast<const float4*>(sh.acc[4 * t + i]);
+            const float gg[4] = {g.x, g.y, g.z, g.w};
+#pragma unroll
+            for (int cc = 0; cc < 4; ++cc)
+                x0[cc][i] = __fadd_rn(x0[cc][i], n == 1 ? gg[cc] : __fdiv_rn(gg[cc], (float)n));
+        }
+    }
+    if (slot < 0 || args.write_anchor_rows) {
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+            if (cc >= cn) break;
+            Lat4<float>::store(args.x0_out, view_base + (size_t)(c.cg + cc) * plane, cnt, VEC, x0[cc]);
+        }
+    }
+    if (recon) {
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+            if (cc >= cn) break;
+            float x[4], y[4], pr[4];
+            Lat4<T>::unpack(xt[cc], x);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) y[i] = recon_one(args.coef, x[i], x0[cc][i], pr[i]);
+            const size_t e = view_base + (size_t)(c.cg + cc) * plane;
+            Lat4<T>::store(xn_p, e, cnt, VEC, y);
+            if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, VEC, pr);
+        }
+    }
+}
 
+// Sparse mode, kernel 1: apply the step's rows of G_{A->v} record-parallel.
+// One thread per record of a pair (v outside the anchor set, anchor u): the
+// kept taps and weights of the record, then the tap-weighted anchor
+// increment sum_k w_k (x0_new - x0(t-1))[q_k] for every channel, written to
+// workspace[r * C + c].  blockIdx.y enumerates (b, view outside A, anchor).
+template <int K>
+__global__ void __launch_bounds__(kThreads) sparse_apply_kernel(const TransportArgs args) {
+    const int N = args.N, C = args.C, a = args.a;
+    const int HW = args.H * args.W;
+    const int T = tiles_per_view_dev(args.H, args.W);
+    const int y = blockIdx.y;
+    const int s2 = y % a;
+    const int vi = (y / a) % (N - a);
+    const int b = y / (a * (N - a));
+    int v = -1;
+    for (int x = 0, r = 0; x < N; ++x)
+        if (args.slot_of[x] < 0 && r++ == vi) { v = x; break; }
+    const int u = args.anchors[s2];
+    const size_t pair = ((size_t)b * N + v) * N + u;
+    const int r0 = __ldg(args.tile_ptr + pair * T), r1 = __ldg(args.tile_ptr + pair * T + T);
+    const size_t plane = (size_t)HW;
+    const float* xn = args.x0_new + ((size_t)b * a + s2) * C * plane;
+    const float* xp = args.x0_prev + ((size_t)b * N + u) * C * plane;
+    for (int r = r0 + blockIdx.x * kThreads + threadIdx.x; r < r1; r += gridDim.x * kThreads) {
+        const int4 rec = __ldg(reinterpret_cast<const int4*>(args.records) + r);
+        Taps tp;
+        taps_from_record<K>((int)((uint32_t)rec.x >> 28), rec.y, __int_as_float(rec.z), __int_as_float(rec.w),
+                            args.W, tp);
+        float* out = args.workspace + (size_t)r * C;
+        for (int cg = 0; cg < C; cg += 4) {
+            const int cn = C - cg < 4 ? C - cg : 4;
+            float dn[K][4], dp[K][4];
+#pragma unroll
+            for (int kk = 0; kk < K; ++kk)
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    dn[kk][c] = 0.0f;
+                    dp[kk][c] = 0.0f;
+                    if (tp.q[kk] >= 0 && c < cn) {
+                        const size_t e = (size_t)(cg + c) * plane + tp.q[kk];
+                        dn[kk][c] = __ldg(xn + e);
+                        dp[kk][c] = __ldg(xp + e);
+                    }
+                }
+            float g[4];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                float acc = 0.0f;
+#pragma unroll
+                for (int kk = 0; kk < K; ++kk)
+                    if (tp.q[kk] >= 0) acc = __fmaf_rn(tp.w[kk], __fsub_rn(dn[kk][c], dp[kk][c]), acc);
+                g[c] = acc;
+            }
+            if (cn == 4 && C % 4 == 0) {
+                *reinterpret_cast<float4*>(out + cg) = make_float4(g[0], g[1], g[2], g[3]);
+            } else {
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    if (c < cn) out[cg + c] = g[c];
+            }
+        }
+    }
+}
+
+// Sparse mode, kernel 2: one CTA per tile of kTileTokens tokens of a view,
+// thread t streams the quad of tokens 4t..4t+3 (all channels in groups of 4,
+// 16-byte accesses).  For views outside the anchor set the tile's records of
+// every anchor are read back with their increments from the workspace and
+// summed per token in anchor order (deterministic; the mean over covering
+// anchors of Eq. 1 with the aggregation of Sec. 3.2; tokens without a
+// record keep x0(t-1)).  Then x0(t) is stored and reconstructed.
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(kThreads) sparse_stream_kernel(const TransportArgs args) {
+    __shared__ float s_acc[kTileTokens][4];
+    __shared__ uint8_t s_n[kTileTokens];
+    __shared__ int s_r0[GEOCACHE_MAX_VIEWS], s_cnt[GEOCACHE_MAX_VIEWS];
+    const int HW = args.H * args.W;
+    const int T_tiles = tiles_per_view_dev(args.H, args.W);
+    const int tile = blockIdx.x, v = blockIdx.y, b = blockIdx.z;
+    const int tile0 = tile * kTileTokens;
+    const int t = threadIdx.x;
+    const int p0 = tile0 + 4 * t;
+    const int cnt = p0 < HW ? (HW - p0 < 4 ? HW - p0 : 4) : 0;
+    const int N = args.N, C = args.C, a = args.a;
+    const int slot = args.slot_of[v];
+    const size_t plane = (size_t)HW;
+    const size_t view_base = ((size_t)b * N + v) * C * plane + p0;
+    const float* x0_src = slot >= 0 ? args.x0_new + ((size_t)b * a + slot) * C * plane + p0
+                                    : args.x0_prev + ((size_t)b * N + v) * C * plane + p0;
+    const bool recon = args.coef.enabled;
+    const T* xt_p = static_cast<const T*>(args.x_t);
+    T* xn_p = static_cast<T*>(args.x_next);
+
+    int total = 0;
     for (int cg = 0; cg < C; cg += 4) {
         const int cn = C - cg < 4 ? C - cg : 4;
         float x0[4][4];
         typename Lat4<T>::Raw xt[4];
-        // streaming loads of the channel group first
+        if (cnt > 0) {
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            if (c >= cn) break;
-            const size_t e = view_base + (size_t)(cg + c) * plane;
-            if (slot >= 0)
-                f4_load_keep(args.x0_new, (((size_t)b * a + slot) * C + cg + c) * plane + p0, cnt, VEC, x0[c]);
-            else
-                Lat4<float>::load(args.x0_prev, e, cnt, VEC, x0[c]);
-            if (recon) xt[c] = Lat4<T>::load_raw(xt_p, e, cnt, VEC);
+            for (int c = 0; c < 4; ++c) {
+                if (c >= cn) break;
+                if (slot >= 0)
+                    f4_load_keep(x0_src, (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
+                else
+                    Lat4<float>::load(x0_src, (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
+                if (recon) xt[c] = Lat4<T>::load_raw(xt_p, view_base + (size_t)(cg + c) * plane, cnt, VEC);
+            }
         }
         if (slot < 0) {
-            if (any_cover) {
-#pragma unroll 1
-                for (int i = 0; i < 4; ++i) {
-                    if (!((any_cover >> (8 * i)) & 0xff)) continue;
-                    const int p = p0 + i;
-                    float X0 = 0.f, X1 = 0.f, X2 = 0.f;
-                    if (MODE != GEOCACHE_CORR_TABLE) {
-                        X0 = __ldg(args.pos + 3 * (tv + i));
-                        X1 = __ldg(args.pos + 3 * (tv + i) + 1);
-                        X2 = __ldg(args.pos + 3 * (tv + i) + 2);
+            if (cg == 0 && t < a) {
+                const size_t i = (((size_t)b * N + v) * N + args.anchors[t]) * T_tiles + tile;
+                const int r0 = __ldg(args.tile_ptr + i);
+                s_r0[t] = r0;
+                s_cnt[t] = __ldg(args.tile_ptr + i + 1) - r0;
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                *reinterpret_cast<float4*>(s_acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
+                s_n[4 * t + i] = 0;
+            }
+            __syncthreads();
+            if (cg == 0)
+                for (int s2 = 0; s2 < a; ++s2) total += s_cnt[s2];
+            for (int j0 = 0; j0 < total; j0 += kThreads) {
+                const int j = j0 + t;
+                int s_mine = -1, lp = 0;
+                float g[4] = {0.f, 0.f, 0.f, 0.f};
+                if (j < total) {
+                    int s2 = 0, jj = j;
+                    while (jj >= s_cnt[s2]) jj -= s_cnt[s2++];
+                    const int r = s_r0[s2] + jj;
+                    lp = (__ldg(&args.records[r].token_mask) & 0x0fffffff) - tile0;
+                    const float* w = args.workspace + (size_t)r * C + cg;
+                    if (cn == 4 && C % 4 == 0) {
+                        const float4 q = __ldg(reinterpret_cast<const float4*>(w));
+                        g[0] = q.x; g[1] = q.y; g[2] = q.z; g[3] = q.w;
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 4; ++c)
+                            if (c < cn) g[c] = __ldg(w + c);
                     }
-                    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-                    int n = 0;
-                    for (int s = 0; s < a; ++s) {
-                        const int u = args.anchors[s];
-                        Taps tp;
-                        if (MODE == GEOCACHE_CORR_TABLE) {
-                            const size_t row = (((size_t)b * N + v) * N + u) * plane + p;
-                            tp.kept = 0;
-#pragma unroll
-                            for (int k = 0; k < K; ++k) {
-                                tp.q[k] = __ldg(args.idx + row * K + k);
-                                tp.w[k] = __ldg(args.w + row * K + k);
-                                tp.kept += tp.q[k] >= 0;
-                            }
-                        } else {
-                            const geocache_camera& cam = args.cams[(size_t)b * N + u];
-                            if (MODE == GEOCACHE_CORR_MASK) {
-                                const int m = __ldg(args.keep + (((size_t)b * N + v) * N + u) * plane + p);
-                                if (!m) continue;
-                                Footprint f;
-                                footprint<K>(cam, X0, X1, X2, args.H, args.W, f);
-                                taps_from_mask<K>(f, m, args.W, tp);
-                            } else {
-                                const size_t su = ((size_t)b * N + u) * plane;
-                                compute_taps<K>(cam, args.pos + 3 * su, args.valid + su, args.H, args.W, X0, X1, X2,
-                                                tau2, tp);
-                            }
-                        }
-                        if (!tp.kept) continue;
-                        ++n;
-                        const float* xn = args.x0_new + (((size_t)b * a + s) * C + cg) * plane;
-                        const float* xp = args.x0_prev + (((size_t)b * N + u) * C + cg) * plane;
-#pragma unroll
-                        for (int k = 0; k < K; ++k) {
-                            if (tp.q[k] < 0) continue;
-#pragma unroll
-                            for (int c = 0; c < 4; ++c) {
-                                if (c >= cn) break;
-                                const size_t e = (size_t)c * plane + tp.q[k];
-                                acc[c] = __fmaf_rn(tp.w[k], __fsub_rn(__ldg(xn + e), __ldg(xp + e)), acc[c]);
-                            }
-                        }
+                    s_mine = s2;
+                }
+                // combine in anchor order (deterministic): anchor s2 adds in pass s2
+                for (int s2 = 0; s2 < a; ++s2) {
+                    if (s_mine == s2) {
+                        float4* dst = reinterpret_cast<float4*>(s_acc[lp]);
+                        float4 cur = *dst;
+                        cur.x = __fadd_rn(cur.x, g[0]);
+                        cur.y = __fadd_rn(cur.y, g[1]);
+                        cur.z = __fadd_rn(cur.z, g[2]);
+                        cur.w = __fadd_rn(cur.w, g[3]);
+                        *dst = cur;
+                        s_n[lp] += 1;
                     }
-                    if (n) {
-#pragma unroll
-                        for (int c = 0; c < 4; ++c) {
-                            const float g = n == 1 ? acc[c] : __fdiv_rn(acc[c], (float)n);
-#pragma unroll
-                            for (int ii = 0; ii < 4; ++ii)
-                                if (ii == i) x0[c][ii] = __fadd_rn(x0[c][ii], g);
-                        }
-                    }
+                    __syncthreads();
                 }
             }
+            if (cnt > 0) {
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                if (c >= cn) break;
-                Lat4<float>::store(args.x0_out, view_base + (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
-            }
-        } else if (args.write_anchor_rows) {
+                for (int i = 0; i < 4; ++i) {
+                    const int n = s_n[4 * t + i];
+                    if (!n) continue;
+                    const float4 gq = *reinterpret_cast<const float4*>(s_acc[4 * t + i]);
+                    const float gg[4] = {gq.x, gq.y, gq.z, gq.w};
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                if (c >= cn) break;
-                Lat4<float>::store(args.x0_out, view_base + (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
+                    for (int c = 0; c < 4; ++c)
+                        x0[c][i] = __fadd_rn(x0[c][i], n == 1 ? gg[c] : __fdiv_rn(gg[c], (float)n));
+                }
             }
         }
-        if (recon) {
+        if (cnt > 0) {
 #pragma unroll
             for (int c = 0; c < 4; ++c) {
                 if (c >= cn) break;
-                float x[4], y[4], pr[4];
-                Lat4<T>::unpack(xt[c], x);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) y[i] = recon_one(args.coef, x[i], x0[c][i], pr[i]);
                 const size_t e = view_base + (size_t)(cg + c) * plane;
-                Lat4<T>::store(xn_p, e, cnt, VEC, y);
-                if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, VEC, pr);
+                Lat4<float>::store(args.x0_out, e, cnt, VEC, x0[c]);
+                if (recon) {
+                    float x[4], yv[4], pr[4];
+                    Lat4<T>::unpack(xt[c], x);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) yv[i] = recon_one(args.coef, x[i], x0[c][i], pr[i]);
+                    Lat4<T>::store(xn_p, e, cnt, VEC, yv);
+                    if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, VEC, pr);
+                }
             }
         }
+        if (slot < 0 && cg + 4 < C) __syncthreads();  // sums are rewritten by the next channel group
     }
+}
+
+template <typename T, int K>
+static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
+    const int HW = t.H * t.W;
+    if (t.a < t.N) {
+        const int gx = (HW + 4095) / 4096;
+        const long long gy = (long long)t.B * (t.N - t.a) * t.a;
+        if (gy > 65535) return cudaErrorInvalidConfiguration;
+        sparse_apply_kernel<K><<<dim3(gx, (unsigned)gy), kThreads, 0, s>>>(t);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    const uintptr_t al = (uintptr_t)t.x0_new | (uintptr_t)t.x0_prev | (uintptr_t)t.x0_out | (uintptr_t)t.x_t |
+                         (uintptr_t)t.x_next | (uintptr_t)t.pred_out;
+    const bool vec = (HW % 4 == 0) && (al % 16 == 0);
+    dim3 grid((HW + kTileTokens - 1) / kTileTokens, t.N, t.B);
+    if (vec)
+        sparse_stream_kernel<T, true><<<grid, kThreads, 0, s>>>(t);
+    else
+        sparse_stream_kernel<T, false><<<grid, kThreads, 0, s>>>(t);
+    return cudaGetLastError();
+}
+
+// Persistent grid size of an instantiation: resident CTAs per SM x SMs.
+template <typename Kern>
+static int persistent_grid(Kern kern, size_t dyn_smem) {
+    int dev = 0, sms = 0, per_sm = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, dyn_smem) != cudaSuccess) return 0;
+    return sms * (per_sm > 0 ? per_sm : 1);
 }
 
 template <typename T, int K, int MODE>
@@ -427,18 +1133,36 @@ static cudaError_t launch_quad(const TransportArgs& t, cudaStream_t s) {
     const uintptr_t al = (uintptr_t)t.x0_new | (uintptr_t)t.x0_prev | (uintptr_t)t.x0_out | (uintptr_t)t.x_t |
                          (uintptr_t)t.x_next | (uintptr_t)t.pred_out | (uintptr_t)t.keep | (uintptr_t)t.valid;
     const bool vec = (HW % 4 == 0) && (al % 16 == 0);
-    const int quads = (HW + 3) / 4;
-    dim3 grid((quads + kThreads - 1) / kThreads, t.N, t.B);
+    const int n_tiles = (HW + kTileTokens - 1) / kTileTokens;
+    const int n_cg = (t.C + 3) / 4;
+    const long long n_units = (long long)t.B * t.N * n_tiles * n_cg;
+    // TMA bulk rows need 16-byte aligned starts and sizes: HW % 8 == 0 covers bf16 rows
+    if (vec && HW % 8 == 0) {
+        const size_t dyn = kStages * 4 * kTileTokens * (sizeof(float) + sizeof(T));
+        auto kern = transport_fused_kernel<T, K, MODE>;
+        static int grid = 0;  // per instantiation and process (one device per process)
+        if (!grid) {
+            cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+            if (e != cudaSuccess) return e;
+            grid = persistent_grid(kern, dyn);
+            if (!grid) return cudaErrorInvalidConfiguration;
+        }
+        const long long g = n_units < grid ? n_units : grid;
+        kern<<<(unsigned)g, kThreads, dyn, s>>>(t, n_tiles, n_cg, n_units);
+        return cudaGetLastError();
+    }
+    if (n_units > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     if (vec)
-        transport_quad_kernel<T, K, MODE, true><<<grid, kThreads, 0, s>>>(t);
+        transport_simple_kernel<T, K, MODE, true><<<(unsigned)n_units, kThreads, 0, s>>>(t, n_tiles, n_cg);
     else
-        transport_quad_kernel<T, K, MODE, false><<<grid, kThreads, 0, s>>>(t);
+        transport_simple_kernel<T, K, MODE, false><<<(unsigned)n_units, kThreads, 0, s>>>(t, n_tiles, n_cg);
     return cudaGetLastError();
 }
 
 template <typename T, int K>
 static cudaError_t launch_transport_t(const TransportArgs& t, cudaStream_t s) {
     switch (t.mode) {
+        case GEOCACHE_CORR_SPARSE: return launch_sparse<T, K>(t, s);
         case GEOCACHE_CORR_MASK: return launch_quad<T, K, GEOCACHE_CORR_MASK>(t, s);
         case GEOCACHE_CORR_TABLE: return launch_quad<T, K, GEOCACHE_CORR_TABLE>(t, s);
         default: return launch_quad<T, K, GEOCACHE_CORR_GEOMETRY>(t, s);
@@ -517,6 +1241,17 @@ cudaError_t launch_reconstruct(const void* x_t, const float* x0, void* x_next, i
     if (lat_dtype == GEOCACHE_BF16)
         return launch_reconstruct_t<__nv_bfloat16>(x_t, x0, x_next, n, coef, pred_out, x0_store, s);
     return launch_reconstruct_t<float>(x_t, x0, x_next, n, coef, pred_out, x0_store, s);
+}
+
+cudaError_t read_device_error(unsigned int* out, bool clear, cudaStream_t s) {
+    cudaError_t e = cudaMemcpyFromSymbolAsync(out, g_device_error, sizeof(unsigned int), 0, cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return e;
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess || !clear || *out == 0) return e;
+    static const unsigned int zero = 0;
+    e = cudaMemcpyToSymbolAsync(g_device_error, &zero, sizeof(unsigned int), 0, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return e;
+    return cudaStreamSynchronize(s);
 }
 
 }  // namespace geocache

@@ -20,7 +20,8 @@ OK, EINVAL, ESHAPE, EDTYPE, ECUDA, ETIMEOUT, EDEVICE, EALIAS = 0, -1, -2, -3, -4
 F32, BF16 = 0, 1
 DDIM, FM_EULER = 0, 1
 PRED_NONE, PRED_EPS, PRED_V, PRED_VELOCITY = 0, 1, 2, 3
-CORR_GEOMETRY, CORR_TABLE, CORR_MASK = 0, 1, 2
+CORR_GEOMETRY, CORR_TABLE, CORR_MASK, CORR_SPARSE = 0, 1, 2, 3
+TILE_TOKENS = 1024
 SCHED_EVERY_K, SCHED_HEAD_MID_TAIL, SCHED_LIST, SCHED_ALL_FULL, SCHED_SINGLE_CACHED = 0, 1, 2, 3, 4
 MAX_VIEWS = 64
 
@@ -45,7 +46,8 @@ class Corr(ctypes.Structure):
                 ("K", ctypes.c_int), ("tol_frac", ctypes.c_float),
                 ("pos", ctypes.c_void_p), ("valid", ctypes.c_void_p), ("cams", ctypes.c_void_p),
                 ("tau", ctypes.c_void_p), ("idx", ctypes.c_void_p), ("w", ctypes.c_void_p),
-                ("keep", ctypes.c_void_p), ("mode", ctypes.c_int)]
+                ("keep", ctypes.c_void_p), ("tile_ptr", ctypes.c_void_p), ("records", ctypes.c_void_p),
+                ("max_records", ctypes.c_int64), ("mode", ctypes.c_int)]
 
 
 class Recon(ctypes.Structure):
@@ -64,7 +66,8 @@ assert ctypes.sizeof(Camera) == 64
 
 _LIB = None
 EXPORTS = ("geocache_build_corr", "geocache_transport_step", "geocache_reconstruct", "geocache_is_full_step",
-           "geocache_rotate_anchors", "geocache_last_error", "geocache_abi_version")
+           "geocache_rotate_anchors", "geocache_device_status", "geocache_corr_record_count",
+           "geocache_transport_workspace", "geocache_last_error", "geocache_abi_version")
 
 
 def lib_path() -> str:
@@ -83,14 +86,19 @@ def load():
         P, i, i64 = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64
         L.geocache_build_corr.argtypes = [ctypes.POINTER(Corr), P]
         L.geocache_transport_step.argtypes = [ctypes.POINTER(Corr), P, i, i, P, P, P, P, P, i,
-                                              ctypes.POINTER(Recon), P]
+                                              ctypes.POINTER(Recon), P, i64, P]
+        L.geocache_corr_record_count.argtypes = [ctypes.POINTER(Corr), ctypes.POINTER(ctypes.c_int64), P]
+        L.geocache_corr_record_count.restype = ctypes.c_int
+        L.geocache_transport_workspace.argtypes = [ctypes.POINTER(Corr), i]
+        L.geocache_transport_workspace.restype = ctypes.c_int64
         L.geocache_reconstruct.argtypes = [P, P, P, i, i64, ctypes.POINTER(Recon), P, P]
         L.geocache_is_full_step.argtypes = [i, i, ctypes.POINTER(Schedule)]
         L.geocache_rotate_anchors.argtypes = [i, i, i, i, ctypes.POINTER(Schedule), P, ctypes.POINTER(i)]
+        L.geocache_device_status.argtypes = [P]
         L.geocache_last_error.restype = ctypes.c_char_p
         L.geocache_last_error.argtypes = []
         L.geocache_abi_version.argtypes = []
-        for name in EXPORTS[:5]:
+        for name in EXPORTS[:7]:
             getattr(L, name).restype = ctypes.c_int
         L.geocache_abi_version.restype = ctypes.c_int
         _LIB = L
@@ -163,22 +171,66 @@ class CorrHandle:
     def keep(self):
         return self._keep.get("keep")
 
+    def workspace_floats(self, C: int) -> int:
+        return load().geocache_transport_workspace(ctypes.byref(self.c), int(C))
 
-def make_corr(pos, valid, cams, tau, idx=None, w=None, K=4, tol_frac=0.01, mode=None, keep=None) -> CorrHandle:
-    """Describe a batch's geometry (and optional tables / keep masks) for the
-    C ABI.  The default mode is MASK when keep masks are given, else TABLE
-    when tables are given, else GEOMETRY."""
+
+def tiles_per_view(H: int, W: int) -> int:
+    return -(-(H * W) // TILE_TOKENS)
+
+
+def make_corr(pos, valid, cams, tau, idx=None, w=None, K=4, tol_frac=0.01, mode=None, keep=None,
+              tile_ptr=None, records=None) -> CorrHandle:
+    """Describe a batch's geometry (and optional tables, keep masks and sparse
+    form) for the C ABI.  records is an int32 tensor [R, 4] (16-byte tap
+    records).  The default mode is SPARSE when records are given, else MASK
+    when keep masks are given, else TABLE when tables are given, else GEOMETRY."""
     B, N, H, W = valid.shape
     n = B * N * H * W
-    refs = {"pos": pos, "valid": valid, "cams": cams, "tau": tau, "idx": idx, "w": w, "keep": keep}
+    refs = {"pos": pos, "valid": valid, "cams": cams, "tau": tau, "idx": idx, "w": w, "keep": keep,
+            "tile_ptr": tile_ptr, "records": records}
     if mode is None:
-        mode = CORR_MASK if keep is not None else (CORR_TABLE if idx is not None else CORR_GEOMETRY)
+        mode = (CORR_SPARSE if records is not None else CORR_MASK if keep is not None
+                else CORR_TABLE if idx is not None else CORR_GEOMETRY)
+    if records is not None and (records.dim() != 2 or records.shape[1] != 4):
+        raise ValueError("records must be an int32 tensor of shape [R, 4]")
     c = Corr(B, N, H, W, K, tol_frac,
              _dev(pos, torch.float32, 3 * n, "pos"), _dev(valid, torch.uint8, n, "valid"),
              _dev(cams, torch.float32, 16 * B * N, "cams"), _dev(tau, torch.float32, B, "tau"),
              _dev(idx, torch.int32, n * N * K, "idx"), _dev(w, torch.float32, n * N * K, "w"),
-             _dev(keep, torch.uint8, n * N, "keep"), mode)
+             _dev(keep, torch.uint8, n * N, "keep"),
+             _dev(tile_ptr, torch.int32, B * N * N * tiles_per_view(H, W) + 1, "tile_ptr"),
+             _dev(records, torch.int32, None, "records"), 0 if records is None else records.shape[0], mode)
     return CorrHandle(c, refs)
+
+
+def record_count(corr: CorrHandle, stream=None) -> int:
+    """geocache_corr_record_count (synchronous)."""
+    n = ctypes.c_int64(0)
+    _check(load().geocache_corr_record_count(ctypes.byref(corr.c), ctypes.byref(n), _stream(stream)))
+    return int(n.value)
+
+
+def build_sparse_corr(pos, valid, cams, K=4, tol_frac=0.01, tables=False, stream=None) -> CorrHandle:
+    """Allocate and build the full correspondence state of a batch: tau, keep
+    masks, the sparse form (count, then records) and optionally the tables.
+    Allocation happens here, once per batch of assets, never per step."""
+    B, N, H, W = valid.shape
+    dev = pos.device
+    tau = torch.zeros(B, dtype=torch.float32, device=dev)
+    keep = torch.empty((B, N, N, H, W), dtype=torch.uint8, device=dev)
+    tile_ptr = torch.empty(B * N * N * tiles_per_view(H, W) + 1, dtype=torch.int32, device=dev)
+    c0 = make_corr(pos, valid, cams, tau, K=K, tol_frac=tol_frac, keep=keep, tile_ptr=tile_ptr,
+                   mode=CORR_MASK)
+    R = record_count(c0, stream)
+    records = torch.empty((max(R, 1), 4), dtype=torch.int32, device=dev)
+    idx = w = None
+    if tables:
+        idx = torch.empty((B, N, N, H, W, K), dtype=torch.int32, device=dev)
+        w = torch.empty((B, N, N, H, W, K), dtype=torch.float32, device=dev)
+    corr = make_corr(pos, valid, cams, tau, idx=idx, w=w, K=K, tol_frac=tol_frac, keep=keep, tile_ptr=tile_ptr,
+                     records=records, mode=CORR_SPARSE)
+    return build_corr(corr, stream)
 
 
 def make_recon(sampler="ddim", a_t=0.0, a_prev=0.0, sigma=0.0, sigma_next=0.0, pred_kind=None,
@@ -216,7 +268,7 @@ def build_corr(corr: CorrHandle, stream=None) -> CorrHandle:
 
 
 def transport_step(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev, x0_out, x_t=None, x_next=None,
-                   recon: Recon | None = None, stream=None):
+                   recon: Recon | None = None, workspace=None, stream=None):
     """geocache_transport_step on torch tensors (see include/geocache.h)."""
     c = corr.c
     anc = sorted(int(a) for a in anchors)
@@ -234,7 +286,9 @@ def transport_step(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev, x0_out,
         ctypes.byref(c), ctypes.cast(arr, ctypes.c_void_p), a, int(C),
         _dev(x0_anchor_new, torch.float32, c.B * a * C * c.H * c.W, "x0_anchor_new"),
         _dev(x0_prev, torch.float32, n_all, "x0_prev"), _dev(x0_out, torch.float32, n_all, "x0_out"),
-        pt, pn, lat, ctypes.byref(recon) if recon is not None else None, _stream(stream))
+        pt, pn, lat, ctypes.byref(recon) if recon is not None else None,
+        _dev(workspace, torch.float32, None, "workspace"), 0 if workspace is None else workspace.numel(),
+        _stream(stream))
     _check(st)
 
 
@@ -266,12 +320,20 @@ def rotate_anchors(N: int, a: int, step: int, S: int, sched: dict):
     return list(out), bool(full.value)
 
 
-def transport_launches(a: int, C: int, in_place: bool = False) -> int:
-    """Kernels one geocache_transport_step enqueues: the tiled kernel for
-    a <= 8 anchors (else one per group of 16 channels), plus the anchor-row
+def transport_launches(a: int, N: int, mode: int, in_place: bool = False) -> int:
+    """Kernels one geocache_transport_step enqueues: sparse mode runs the
+    record-parallel apply (when some view is outside the anchor set) and the
+    streaming kernel; the other modes one fused kernel, plus the anchor-row
     copy of an in-place update."""
-    n = 1 if a <= 8 else -(-C // (4 if C <= 4 else 16))
-    return n + (1 if in_place else 0)
+    if mode == CORR_SPARSE:
+        return 2 if a < N else 1
+    return 1 + (1 if in_place else 0)
+
+
+def device_status(stream=None):
+    """geocache_device_status: raise GeocacheError(ETIMEOUT) if a kernel's
+    bounded wait gave up since the last check."""
+    _check(load().geocache_device_status(_stream(stream)))
 
 
 def abi_version() -> int:

@@ -126,12 +126,24 @@ class DeviceGeometry:
             self.idx = torch.empty(shp, dtype=torch.int32, device=dev)
             self.wt = torch.empty(shp, dtype=torch.float32, device=dev)
         self.keep = torch.empty((w.B, w.N, w.N, w.H, w.W), dtype=torch.uint8, device=dev)
+        self.tile_ptr = torch.empty(w.B * w.N * w.N * gc.tiles_per_view(w.H, w.W) + 1, dtype=torch.int32,
+                                    device=dev)
+        c0 = gc.make_corr(self.pos, self.valid, self.cams, self.tau, K=K, tol_frac=w.tol_frac, keep=self.keep,
+                          tile_ptr=self.tile_ptr, mode=gc.CORR_MASK)
+        self.n_records = gc.record_count(c0)
+        self.records = torch.empty((max(self.n_records, 1), 4), dtype=torch.int32, device=dev)
         self.corr = gc.make_corr(self.pos, self.valid, self.cams, self.tau, self.idx, self.wt, K=K,
-                                 tol_frac=w.tol_frac, keep=self.keep, mode=gc.CORR_MASK)
+                                 tol_frac=w.tol_frac, keep=self.keep, tile_ptr=self.tile_ptr, records=self.records,
+                                 mode=gc.CORR_SPARSE)
         gc.build_corr(self.corr)
 
     def corr_for(self, mode):
         gc = self.gc
-        m = {"mask": gc.CORR_MASK, "geometry": gc.CORR_GEOMETRY, "table": gc.CORR_TABLE}[mode]
+        m = {"mask": gc.CORR_MASK, "geometry": gc.CORR_GEOMETRY, "table": gc.CORR_TABLE,
+             "sparse": gc.CORR_SPARSE}[mode]
         return gc.make_corr(self.pos, self.valid, self.cams, self.tau, self.idx, self.wt, K=self.K,
-                            tol_frac=self.w.tol_frac, keep=self.keep, mode=m)
+                            tol_frac=self.w.tol_frac, keep=self.keep, tile_ptr=self.tile_ptr, records=self.records,
+                            mode=m)
+
+    def workspace(self, C):
+        return torch.empty(max(self.corr.workspace_floats(C), 4), dtype=torch.float32, device=self.pos.device)

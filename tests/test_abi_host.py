@@ -77,27 +77,38 @@ def test_tiny_first_cached_step_anchors(gc):
 def test_argument_errors_before_launch(gc):
     L = gc.load()
     # NULL corr, bad sizes, bad anchors, bad sampler: rejected on the host
-    assert L.geocache_transport_step(None, None, 0, 0, None, None, None, None, None, 0, None, None) == gc.EINVAL
+    assert L.geocache_transport_step(None, None, 0, 0, None, None, None, None, None, 0, None, None, 0, None) == gc.EINVAL
     assert "corr" in gc.last_error()
     c = gc.Corr(1, 6, 8, 8, 4, 0.01, 16, 16, 16, 16, None, None, None, gc.CORR_GEOMETRY)
     anc = (ctypes.c_int32 * 2)(3, 0)  # not ascending
     st = L.geocache_transport_step(ctypes.byref(c), ctypes.cast(anc, ctypes.c_void_p), 2, 4, 16, 16, 32,
-                                   None, None, 0, None, None)
+                                   None, None, 0, None, None, 0, None)
     assert st == gc.EINVAL and "ascending" in gc.last_error()
     anc = (ctypes.c_int32 * 2)(0, 3)
     st = L.geocache_transport_step(ctypes.byref(c), ctypes.cast(anc, ctypes.c_void_p), 2, 0, 16, 16, 32,
-                                   None, None, 0, None, None)
+                                   None, None, 0, None, None, 0, None)
     assert st == gc.ESHAPE
     c.K = 3
     st = L.geocache_transport_step(ctypes.byref(c), ctypes.cast(anc, ctypes.c_void_p), 2, 4, 16, 16, 32,
-                                   None, None, 0, None, None)
+                                   None, None, 0, None, None, 0, None)
     assert st == gc.EINVAL
     c.K = 4
     c.mode = gc.CORR_MASK  # mask mode without keep masks
     st = L.geocache_transport_step(ctypes.byref(c), ctypes.cast(anc, ctypes.c_void_p), 2, 4, 16, 16, 32,
-                                   None, None, 0, None, None)
+                                   None, None, 0, None, None, 0, None)
     assert st == gc.EINVAL and "keep" in gc.last_error()
+    c.mode = gc.CORR_SPARSE  # sparse mode without records / workspace
+    st = L.geocache_transport_step(ctypes.byref(c), ctypes.cast(anc, ctypes.c_void_p), 2, 4, 16, 16, 32,
+                                   None, None, 0, None, None, 0, None)
+    assert st == gc.EINVAL and "tile_ptr" in gc.last_error()
+    c.tile_ptr, c.records, c.max_records = 64, 128, 10
+    st = L.geocache_transport_step(ctypes.byref(c), ctypes.cast(anc, ctypes.c_void_p), 2, 4, 16, 16, 32,
+                                   None, None, 0, None, None, 0, None)
+    assert st == gc.EINVAL and "workspace" in gc.last_error()
+    assert L.geocache_transport_workspace(ctypes.byref(c), 4) == 40
+    c.tile_ptr, c.records, c.max_records = None, None, 0
     c.mode = gc.CORR_GEOMETRY
+    assert L.geocache_transport_workspace(ctypes.byref(c), 4) == 0
     c.N = 65
     assert L.geocache_build_corr(ctypes.byref(c), None) == gc.ESHAPE
     c.N = 6

@@ -47,6 +47,26 @@ def _compare_tables(w, g, K):
     keep_ref = sum((kept[..., k].astype(np.uint8) << k) for k in range(K))
     keep = g.keep.cpu().numpy()
     assert not ((keep != keep_ref) & (band == 0)).any(), "keep masks differ outside the threshold band"
+    # sparse form: one record per kept row, in (b, v, u, token) order, whose
+    # taps are the table's taps
+    if not band.any():
+        rec = g.records.cpu().numpy()[: g.n_records]
+        tp = g.tile_ptr.cpu().numpy()
+        T = g.gc.tiles_per_view(w.H, w.W)
+        rows = np.flatnonzero(keep_ref.reshape(-1) > 0)  # (b, v, u, p) order
+        assert g.n_records == len(rows) == tp[-1]
+        HW = w.H * w.W
+        p = rows % HW
+        assert (rec[:, 0] & 0x0FFFFFFF == p).all()
+        assert ((rec[:, 0] >> 28) & 15 == keep_ref.reshape(-1)[rows]).all()
+        pair = rows // HW
+        counts = np.bincount(pair * T + p // 1024, minlength=w.B * w.N * w.N * T)
+        np.testing.assert_array_equal(tp, np.concatenate([[0], np.cumsum(counts)]))
+        q_tl = rec[:, 1].astype(np.int64)
+        ir = idx_ref.reshape(-1, K)[rows]
+        offs = np.array([0, 1, w.W, w.W + 1])[:K] if K == 4 else np.array([0])
+        expect = np.where(ir >= 0, q_tl[:, None] + offs[None, :], -1)
+        np.testing.assert_array_equal(expect, ir)
     return int(band.sum()), float(kept.any(-1).mean())
 
 
@@ -67,7 +87,7 @@ def test_tables_bit_exact_k1(gc, workloads, name):
     _compare_tables(w, g, 1)
 
 
-def _run_step(gc, w, g, anchors, params, pred=None, mode="mask", inplace=False, xinplace=False,
+def _run_step(gc, w, g, anchors, params, pred=None, mode="sparse", inplace=False, xinplace=False,
               seed_extra=0, C=None):
     """One cached step on the GPU and in the oracle from the same inputs."""
     if C is not None and C != w.C:
@@ -85,8 +105,9 @@ def _run_step(gc, w, g, anchors, params, pred=None, mode="mask", inplace=False, 
     r = gc.make_recon(params["sampler"], a_t=params.get("a_t", 0), a_prev=params.get("a_prev", 0),
                       sigma=params.get("sigma", 0), sigma_next=params.get("sigma_next", 0),
                       pred_kind=pred, pred_out=d_pred)
-    gc.transport_step(corr, anchors, w.C, d_new, d_prev, d_out, d_xt, d_xn, r)
+    gc.transport_step(corr, anchors, w.C, d_new, d_prev, d_out, d_xt, d_xn, r, workspace=g.workspace(w.C))
     torch.cuda.synchronize()
+    gc.device_status()
     tau_ref = oracle.tau(w.pos, w.valid, w.tol_frac)
     ref_x0, ref_xn, ref_pred = oracle.transport_step(
         anchors, x0_new, x0_prev, K=g.corr.c.K, geom=(w.pos, w.valid, w.cams, tau_ref), x_t=xt64,
@@ -129,12 +150,15 @@ def test_transport_step_parity(gc, workloads, name):
 
 @pytest.mark.parametrize("name,K", [("hunyuan64", 4), ("ring12_128", 4), ("solids96", 1)])
 def test_corr_modes_agree_bitwise(gc, workloads, name, K):
-    # keep masks, full geometry and tables give the same taps and weights
+    # sparse records, keep masks, full geometry and tables give the same
+    # taps, weights and results
     w = workloads(name)
     g = DeviceGeometry(w, K=K)
     anchors = oracle.rotate_anchors(w.N, w.a, 1)
     params = synth.recon_params(w, 7)
+    _, _, got_sparse, _ = _run_step(gc, w, g, anchors, params, mode="sparse")
     _, _, got_mask, _ = _run_step(gc, w, g, anchors, params, mode="mask")
+    np.testing.assert_array_equal(got_sparse, got_mask)
     _, _, got_geom, _ = _run_step(gc, w, g, anchors, params, mode="geometry")
     _, _, got_tab, _ = _run_step(gc, w, g, anchors, params, mode="table")
     np.testing.assert_array_equal(got_mask, got_geom)
@@ -162,8 +186,9 @@ def test_in_place_cache_and_latents(gc, workloads):
     g = DeviceGeometry(w, K=4, tables=False)
     params = synth.recon_params(w, 4)
     _, _, a, _ = _run_step(gc, w, g, [1, 4], params)
-    _, _, b, _ = _run_step(gc, w, g, [1, 4], params, inplace=True, xinplace=True)
-    np.testing.assert_array_equal(a, b)
+    for mode in ("sparse", "mask"):
+        _, _, b, _ = _run_step(gc, w, g, [1, 4], params, inplace=True, xinplace=True, mode=mode)
+        np.testing.assert_array_equal(a, b)
 
 
 @pytest.mark.parametrize("C", [1, 3, 5, 16, 20, 33])
@@ -224,7 +249,7 @@ def test_zero_delta_bit_identical(gc, workloads):
     d_prev = torch.from_numpy(x0_prev).cuda()
     d_new = d_prev[:, [0, 3, 6, 9]].contiguous()
     d_out = torch.empty_like(d_prev)
-    gc.transport_step(g.corr, [0, 3, 6, 9], w.C, d_new, d_prev, d_out)
+    gc.transport_step(g.corr, [0, 3, 6, 9], w.C, d_new, d_prev, d_out, workspace=g.workspace(w.C))
     torch.cuda.synchronize()
     assert torch.equal(d_out, d_prev)
 
@@ -240,7 +265,8 @@ def test_all_anchor_step_equals_full_step(gc, workloads):
     r = gc.make_recon("ddim", a_t=p["a_t"], a_prev=p["a_prev"])
     d_new = torch.from_numpy(x0_new).cuda()
     out1, xn1 = torch.empty_like(d_new), torch.empty_like(xt)
-    gc.transport_step(g.corr, list(range(w.N)), w.C, d_new, torch.from_numpy(x0_prev).cuda(), out1, xt, xn1, r)
+    gc.transport_step(g.corr, list(range(w.N)), w.C, d_new, torch.from_numpy(x0_prev).cuda(), out1, xt, xn1, r,
+                      workspace=g.workspace(w.C))
     xn2 = torch.empty_like(xt)
     gc.reconstruct(xt, d_new, xn2, r)
     torch.cuda.synchronize()
@@ -281,6 +307,7 @@ def test_trajectory_per_step_parity_and_drift(gc, workloads):
     reported."""
     w = workloads("hunyuan64")
     g = DeviceGeometry(w, K=4, tables=False)
+    ws = g.workspace(w.C)
     xT, x0_init = synth.initial_latents(w)
     tau_ref = oracle.tau(w.pos, w.valid)
     geom = (w.pos, w.valid, w.cams, tau_ref)
@@ -313,7 +340,7 @@ def test_trajectory_per_step_parity_and_drift(gc, workloads):
             d_new = torch.from_numpy(x0_new).cuda()
             out = torch.empty_like(cache)
             xn = torch.empty_like(x)
-            gc.transport_step(g.corr, anchors, w.C, d_new, cache, out, x, xn, r)
+            gc.transport_step(g.corr, anchors, w.C, d_new, cache, out, x, xn, r, workspace=ws)
             ref_x0, ref_xn, _ = oracle.transport_step(anchors, x0_new, cache.cpu().numpy(), geom=geom,
                                                       x_t=x_in64, recon=rk)
             torch.cuda.synchronize()
