@@ -903,30 +903,111 @@ __global__ void __launch_bounds__(kThreads) transport_simple_kernel(const Transp
     }
 }
 
-// Sparse mode, kernel 1: apply the step's rows of G_{A->v} record-parallel.
-// One thread per record of a pair (v outside the anchor set, anchor u): the
-// kept taps and weights of the record, then the tap-weighted anchor
-// increment sum_k w_k (x0_new - x0(t-1))[q_k] for every channel, written to
-// workspace[r * C + c].  blockIdx.y enumerates (b, view outside A, anchor).
+// Sparse mode.  A cached step is two kernels:
+//  phase A: (i) the records of the step's pairs (v outside the anchor set,
+//    anchor u) applied record-parallel: for each record the kept taps and
+//    weights, then sum_k w_k (x0_new - x0(t-1))[q_k] for every channel,
+//    written to workspace[r * C + c];  (ii) the anchor views streamed
+//    (x0(t) = the denoiser's x0, reconstruction).  The two kinds of CTA are
+//    interleaved in launch order so that the latency-bound gathers overlap
+//    the bandwidth-bound streaming and both read the anchors' fresh x0 while
+//    it is in L2.  For an in-place cache update the anchor rows are written
+//    by phase B instead (the gathers read x0(t-1) of the anchors).
+//  phase B: the other views streamed; each CTA folds its tile's record
+//    increments in anchor order (deterministic: the mean over covering
+//    anchors of Eq. 1 with the aggregation of Sec. 3.2; tokens without a
+//    record keep x0(t-1)), then stores and reconstructs every token.
+
+// Streamed rows of the quad of tokens p0.. of view v of asset b, channel
+// group cg: x0 (the anchor's fresh x0 or x0(t-1)) and x_t.
+template <typename T, bool VEC>
+struct QuadRows {
+    float x0[4][4];
+    typename Lat4<T>::Raw xt[4];
+
+    __device__ __forceinline__ void load(const TransportArgs& args, int b, int v, int slot, int p0, int cnt, int cg,
+                                         int cn) {
+        const size_t plane = (size_t)args.H * args.W;
+        const int N = args.N, C = args.C, a = args.a;
+        const float* x0_src = slot >= 0 ? args.x0_new + ((size_t)b * a + slot) * C * plane + p0
+                                        : args.x0_prev + ((size_t)b * N + v) * C * plane + p0;
+        const T* xt_p = static_cast<const T*>(args.x_t) + ((size_t)b * N + v) * C * plane + p0;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            if (c >= cn) break;
+            if (slot >= 0)
+                f4_load_keep(x0_src, (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
+            else
+                Lat4<float>::load(x0_src, (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
+            if (args.coef.enabled) xt[c] = Lat4<T>::load_raw(xt_p, (size_t)(cg + c) * plane, cnt, VEC);
+        }
+    }
+
+    // add the folded increments of the tile (mean over covering anchors)
+    __device__ __forceinline__ void fold(const float (*s_acc)[4], const uint8_t* s_n, int lp0) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int n = s_n[lp0 + i];
+            if (!n) continue;
+            const float4 gq = *reinterpret_cast<const float4*>(s_acc[lp0 + i]);
+            const float gg[4] = {gq.x, gq.y, gq.z, gq.w};
+#pragma unroll
+            for (int c = 0; c < 4; ++c) x0[c][i] = __fadd_rn(x0[c][i], n == 1 ? gg[c] : __fdiv_rn(gg[c], (float)n));
+        }
+    }
+
+    // store x0(t) and the reconstruction
+    __device__ __forceinline__ void store(const TransportArgs& args, int b, int v, int p0, int cnt, int cg, int cn) {
+        const size_t plane = (size_t)args.H * args.W;
+        const size_t view_base = ((size_t)b * args.N + v) * args.C * plane + p0;
+        T* xn_p = static_cast<T*>(args.x_next);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            if (c >= cn) break;
+            const size_t e = view_base + (size_t)(cg + c) * plane;
+            Lat4<float>::store(args.x0_out, e, cnt, VEC, x0[c]);
+            if (args.coef.enabled) {
+                float x[4], yv[4], pr[4];
+                Lat4<T>::unpack(xt[c], x);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) yv[i] = recon_one(args.coef, x[i], x0[c][i], pr[i]);
+                Lat4<T>::store(xn_p, e, cnt, VEC, yv);
+                if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, VEC, pr);
+            }
+        }
+    }
+};
+
+// Programmatic dependent launch: the dependent grid may start once every CTA
+// of this grid has issued launch_dependents; griddepcontrol.wait blocks until
+// the prerequisite grid has completed and its writes are visible.
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// the v-th view outside the anchor set
+__device__ __forceinline__ int nonanchor_view(const TransportArgs& args, int vi) {
+    for (int x = 0, r = 0; x < args.N; ++x)
+        if (args.slot_of[x] < 0 && r++ == vi) return x;
+    return -1;
+}
+
+// Records of one pair applied by one CTA slice (grid-stride over the pair's records).
 template <int K>
-__global__ void __launch_bounds__(kThreads) sparse_apply_kernel(const TransportArgs args) {
+__device__ __forceinline__ void apply_records(const TransportArgs& args, int pair_id, int slice, int n_slices) {
     const int N = args.N, C = args.C, a = args.a;
     const int HW = args.H * args.W;
     const int T = tiles_per_view_dev(args.H, args.W);
-    const int y = blockIdx.y;
-    const int s2 = y % a;
-    const int vi = (y / a) % (N - a);
-    const int b = y / (a * (N - a));
-    int v = -1;
-    for (int x = 0, r = 0; x < N; ++x)
-        if (args.slot_of[x] < 0 && r++ == vi) { v = x; break; }
+    const int s2 = pair_id % a;
+    const int vi = (pair_id / a) % (N - a);
+    const int b = pair_id / (a * (N - a));
+    const int v = nonanchor_view(args, vi);
     const int u = args.anchors[s2];
     const size_t pair = ((size_t)b * N + v) * N + u;
     const int r0 = __ldg(args.tile_ptr + pair * T), r1 = __ldg(args.tile_ptr + pair * T + T);
     const size_t plane = (size_t)HW;
     const float* xn = args.x0_new + ((size_t)b * a + s2) * C * plane;
     const float* xp = args.x0_prev + ((size_t)b * N + u) * C * plane;
-    for (int r = r0 + blockIdx.x * kThreads + threadIdx.x; r < r1; r += gridDim.x * kThreads) {
+    for (int r = r0 + slice * kThreads + threadIdx.x; r < r1; r += n_slices * kThreads) {
         const int4 rec = __ldg(reinterpret_cast<const int4*>(args.records) + r);
         Taps tp;
         taps_from_record<K>((int)((uint32_t)rec.x >> 28), rec.y, __int_as_float(rec.z), __int_as_float(rec.w),
@@ -967,153 +1048,170 @@ __global__ void __launch_bounds__(kThreads) sparse_apply_kernel(const TransportA
     }
 }
 
-// Sparse mode, kernel 2: one CTA per tile of kTileTokens tokens of a view,
-// thread t streams the quad of tokens 4t..4t+3 (all channels in groups of 4,
-// 16-byte accesses).  For views outside the anchor set the tile's records of
-// every anchor are read back with their increments from the workspace and
-// summed per token in anchor order (deterministic; the mean over covering
-// anchors of Eq. 1 with the aggregation of Sec. 3.2; tokens without a
-// record keep x0(t-1)).  Then x0(t) is stored and reconstructed.
+// Phase A: n_apply record-slice CTAs and n_stream anchor-view CTAs (tiles of
+// kTileTokens tokens), interleaved evenly in block order.
+template <typename T, int K, bool VEC>
+__global__ void __launch_bounds__(kThreads) sparse_phase_a_kernel(const TransportArgs args, int n_apply,
+                                                                  int n_stream, int n_slices) {
+    pdl_launch_dependents();
+    const long long total = (long long)n_apply + n_stream;
+    const long long k = blockIdx.x;
+    const int s_before = (int)(k * n_stream / total);
+    const bool is_stream = (int)((k + 1) * n_stream / total) > s_before;
+    if (!is_stream) {
+        const int ai = (int)k - s_before;
+        apply_records<K>(args, ai / n_slices, ai % n_slices, n_slices);
+        return;
+    }
+    const int n_tiles = tiles_per_view_dev(args.H, args.W);
+    const int tile = s_before % n_tiles;
+    const int slot = (s_before / n_tiles) % args.a;
+    const int b = s_before / (n_tiles * args.a);
+    const int v = args.anchors[slot];
+    const int HW = args.H * args.W;
+    const int tile0 = tile * kTileTokens;
+    const int p0 = tile0 + 4 * threadIdx.x;
+    if (p0 >= HW) return;
+    const int cnt = HW - p0 < 4 ? HW - p0 : 4;
+    for (int cg = 0; cg < args.C; cg += 4) {
+        const int cn = args.C - cg < 4 ? args.C - cg : 4;
+        QuadRows<T, VEC> q;
+        q.load(args, b, v, slot, p0, cnt, cg, cn);
+        q.store(args, b, v, p0, cnt, cg, cn);
+    }
+}
+
+// Phase B: one CTA per tile of a view; blockIdx.y < N - a: views outside the
+// anchor set (fold the tile's increments); blockIdx.y >= N - a: anchor views
+// (only for an in-place cache update, see phase A).
 template <typename T, bool VEC>
-__global__ void __launch_bounds__(kThreads) sparse_stream_kernel(const TransportArgs args) {
+__global__ void __launch_bounds__(kThreads) sparse_phase_b_kernel(const TransportArgs args) {
     __shared__ float s_acc[kTileTokens][4];
     __shared__ uint8_t s_n[kTileTokens];
     __shared__ int s_r0[GEOCACHE_MAX_VIEWS], s_cnt[GEOCACHE_MAX_VIEWS];
     const int HW = args.H * args.W;
     const int T_tiles = tiles_per_view_dev(args.H, args.W);
-    const int tile = blockIdx.x, v = blockIdx.y, b = blockIdx.z;
+    const int tile = blockIdx.x, b = blockIdx.z;
+    const int N = args.N, C = args.C, a = args.a;
     const int tile0 = tile * kTileTokens;
     const int t = threadIdx.x;
     const int p0 = tile0 + 4 * t;
     const int cnt = p0 < HW ? (HW - p0 < 4 ? HW - p0 : 4) : 0;
-    const int N = args.N, C = args.C, a = args.a;
-    const int slot = args.slot_of[v];
-    const size_t plane = (size_t)HW;
-    const size_t view_base = ((size_t)b * N + v) * C * plane + p0;
-    const float* x0_src = slot >= 0 ? args.x0_new + ((size_t)b * a + slot) * C * plane + p0
-                                    : args.x0_prev + ((size_t)b * N + v) * C * plane + p0;
-    const bool recon = args.coef.enabled;
-    const T* xt_p = static_cast<const T*>(args.x_t);
-    T* xn_p = static_cast<T*>(args.x_next);
-
+    if ((int)blockIdx.y >= N - a) {  // anchor view, in-place update: after phase A's gathers
+        const int slot = blockIdx.y - (N - a);
+        pdl_wait();
+        if (cnt <= 0) return;
+        for (int cg = 0; cg < C; cg += 4) {
+            const int cn = C - cg < 4 ? C - cg : 4;
+            QuadRows<T, VEC> q;
+            q.load(args, b, args.anchors[slot], slot, p0, cnt, cg, cn);
+            q.store(args, b, args.anchors[slot], p0, cnt, cg, cn);
+        }
+        return;
+    }
+    const int v = nonanchor_view(args, blockIdx.y);
+    // streamed rows first (phase A writes none of them), tile offsets next
+    QuadRows<T, VEC> q;
+    if (cnt > 0) q.load(args, b, v, -1, p0, cnt, 0, C < 4 ? C : 4);
+    if (t < a) {
+        const size_t i = (((size_t)b * N + v) * N + args.anchors[t]) * T_tiles + tile;
+        const int r0 = __ldg(args.tile_ptr + i);
+        s_r0[t] = r0;
+        s_cnt[t] = __ldg(args.tile_ptr + i + 1) - r0;
+    }
+    pdl_wait();  // phase A's workspace writes are complete and visible
+    __syncthreads();
     int total = 0;
+    for (int s2 = 0; s2 < a; ++s2) total += s_cnt[s2];
     for (int cg = 0; cg < C; cg += 4) {
         const int cn = C - cg < 4 ? C - cg : 4;
-        float x0[4][4];
-        typename Lat4<T>::Raw xt[4];
-        if (cnt > 0) {
+        if (cg > 0 && cnt > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                if (c >= cn) break;
-                if (slot >= 0)
-                    f4_load_keep(x0_src, (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
-                else
-                    Lat4<float>::load(x0_src, (size_t)(cg + c) * plane, cnt, VEC, x0[c]);
-                if (recon) xt[c] = Lat4<T>::load_raw(xt_p, view_base + (size_t)(cg + c) * plane, cnt, VEC);
-            }
+        for (int i = 0; i < 4; ++i) {
+            *reinterpret_cast<float4*>(s_acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
+            s_n[4 * t + i] = 0;
         }
-        if (slot < 0) {
-            if (cg == 0 && t < a) {
-                const size_t i = (((size_t)b * N + v) * N + args.anchors[t]) * T_tiles + tile;
-                const int r0 = __ldg(args.tile_ptr + i);
-                s_r0[t] = r0;
-                s_cnt[t] = __ldg(args.tile_ptr + i + 1) - r0;
-            }
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                *reinterpret_cast<float4*>(s_acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
-                s_n[4 * t + i] = 0;
-            }
-            __syncthreads();
-            if (cg == 0)
-                for (int s2 = 0; s2 < a; ++s2) total += s_cnt[s2];
-            for (int j0 = 0; j0 < total; j0 += kThreads) {
-                const int j = j0 + t;
-                int s_mine = -1, lp = 0;
-                float g[4] = {0.f, 0.f, 0.f, 0.f};
-                if (j < total) {
-                    int s2 = 0, jj = j;
-                    while (jj >= s_cnt[s2]) jj -= s_cnt[s2++];
-                    const int r = s_r0[s2] + jj;
-                    lp = (__ldg(&args.records[r].token_mask) & 0x0fffffff) - tile0;
-                    const float* w = args.workspace + (size_t)r * C + cg;
-                    if (cn == 4 && C % 4 == 0) {
-                        const float4 q = __ldg(reinterpret_cast<const float4*>(w));
-                        g[0] = q.x; g[1] = q.y; g[2] = q.z; g[3] = q.w;
-                    } else {
-#pragma unroll
-                        for (int c = 0; c < 4; ++c)
-                            if (c < cn) g[c] = __ldg(w + c);
-                    }
-                    s_mine = s2;
-                }
-                // combine in anchor order (deterministic): anchor s2 adds in pass s2
-                for (int s2 = 0; s2 < a; ++s2) {
-                    if (s_mine == s2) {
-                        float4* dst = reinterpret_cast<float4*>(s_acc[lp]);
-                        float4 cur = *dst;
-                        cur.x = __fadd_rn(cur.x, g[0]);
-                        cur.y = __fadd_rn(cur.y, g[1]);
-                        cur.z = __fadd_rn(cur.z, g[2]);
-                        cur.w = __fadd_rn(cur.w, g[3]);
-                        *dst = cur;
-                        s_n[lp] += 1;
-                    }
-                    __syncthreads();
-                }
-            }
-            if (cnt > 0) {
-#pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int n = s_n[4 * t + i];
-                    if (!n) continue;
-                    const float4 gq = *reinterpret_cast<const float4*>(s_acc[4 * t + i]);
-                    const float gg[4] = {gq.x, gq.y, gq.z, gq.w};
+        __syncthreads();
+        for (int j0 = 0; j0 < total; j0 += kThreads) {
+            const int j = j0 + t;
+            int s_mine = -1, lp = 0;
+            float g[4] = {0.f, 0.f, 0.f, 0.f};
+            if (j < total) {
+                int s2 = 0, jj = j;
+                while (jj >= s_cnt[s2]) jj -= s_cnt[s2++];
+                const int r = s_r0[s2] + jj;
+                lp = (__ldg(&args.records[r].token_mask) & 0x0fffffff) - tile0;
+                const float* w = args.workspace + (size_t)r * C + cg;
+                if (cn == 4 && C % 4 == 0) {
+                    const float4 wq = *reinterpret_cast<const float4*>(w);
+                    g[0] = wq.x; g[1] = wq.y; g[2] = wq.z; g[3] = wq.w;
+                } else {
 #pragma unroll
                     for (int c = 0; c < 4; ++c)
-                        x0[c][i] = __fadd_rn(x0[c][i], n == 1 ? gg[c] : __fdiv_rn(gg[c], (float)n));
+                        if (c < cn) g[c] = w[c];
                 }
+                s_mine = s2;
+            }
+            // combine in anchor order (deterministic): anchor s2 adds in pass s2
+            for (int s2 = 0; s2 < a; ++s2) {
+                if (s_mine == s2) {
+                    float4* dst = reinterpret_cast<float4*>(s_acc[lp]);
+                    float4 cur = *dst;
+                    cur.x = __fadd_rn(cur.x, g[0]);
+                    cur.y = __fadd_rn(cur.y, g[1]);
+                    cur.z = __fadd_rn(cur.z, g[2]);
+                    cur.w = __fadd_rn(cur.w, g[3]);
+                    *dst = cur;
+                    s_n[lp] += 1;
+                }
+                __syncthreads();
             }
         }
         if (cnt > 0) {
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                if (c >= cn) break;
-                const size_t e = view_base + (size_t)(cg + c) * plane;
-                Lat4<float>::store(args.x0_out, e, cnt, VEC, x0[c]);
-                if (recon) {
-                    float x[4], yv[4], pr[4];
-                    Lat4<T>::unpack(xt[c], x);
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) yv[i] = recon_one(args.coef, x[i], x0[c][i], pr[i]);
-                    Lat4<T>::store(xn_p, e, cnt, VEC, yv);
-                    if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, VEC, pr);
-                }
-            }
+            q.fold(s_acc, s_n, 4 * t);
+            q.store(args, b, v, p0, cnt, cg, cn);
         }
-        if (slot < 0 && cg + 4 < C) __syncthreads();  // sums are rewritten by the next channel group
+        if (cg + 4 < C) __syncthreads();  // sums are rewritten by the next channel group
     }
 }
 
 template <typename T, int K>
 static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
     const int HW = t.H * t.W;
-    if (t.a < t.N) {
-        const int gx = (HW + 4095) / 4096;
-        const long long gy = (long long)t.B * (t.N - t.a) * t.a;
-        if (gy > 65535) return cudaErrorInvalidConfiguration;
-        sparse_apply_kernel<K><<<dim3(gx, (unsigned)gy), kThreads, 0, s>>>(t);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
-    }
+    const int n_tiles = (HW + kTileTokens - 1) / kTileTokens;
     const uintptr_t al = (uintptr_t)t.x0_new | (uintptr_t)t.x0_prev | (uintptr_t)t.x0_out | (uintptr_t)t.x_t |
                          (uintptr_t)t.x_next | (uintptr_t)t.pred_out;
     const bool vec = (HW % 4 == 0) && (al % 16 == 0);
-    dim3 grid((HW + kTileTokens - 1) / kTileTokens, t.N, t.B);
-    if (vec)
-        sparse_stream_kernel<T, true><<<grid, kThreads, 0, s>>>(t);
-    else
-        sparse_stream_kernel<T, false><<<grid, kThreads, 0, s>>>(t);
+    const bool in_place = t.x0_out == t.x0_prev;
+    const int n_slices = (HW + 4095) / 4096;
+    const long long n_apply = t.a < t.N ? (long long)t.B * (t.N - t.a) * t.a * n_slices : 0;
+    const long long n_stream = in_place ? 0 : (long long)t.B * t.a * n_tiles;
+    if (n_apply + n_stream > 0) {
+        if (n_apply + n_stream > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+        const unsigned g = (unsigned)(n_apply + n_stream);
+        if (vec)
+            sparse_phase_a_kernel<T, K, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
+        else
+            sparse_phase_a_kernel<T, K, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    const int gy = (t.N - t.a) + (in_place ? t.a : 0);
+    if (gy > 0) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(n_tiles, gy, t.B);
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = 0;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = n_apply + n_stream > 0 ? 1 : 0;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        cudaError_t e = vec ? cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true>, t)
+                            : cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false>, t);
+        if (e != cudaSuccess) return e;
+    }
     return cudaGetLastError();
 }
 
