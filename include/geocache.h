@@ -269,6 +269,33 @@ int geocache_rotate_anchors(int N, int a, int step, int S, const geocache_schedu
  * ------------------------------------------------------------------------ */
 int geocache_device_status(void* stream);
 
+/* --------------------------------------------------------------------------
+ * geocache_transport_step_noalloc -- geocache_transport_step for callers that
+ * cannot supply a workspace (the paper has no counterpart; this is a service
+ * of the library).  Some callers cannot obtain a device buffer where they run
+ * a step: their device memory is owned by another component (a framework's
+ * caching allocator, a fixed arena), or they must not allocate once running
+ * because cudaMalloc can synchronise the device and stall.  This entry point
+ * takes the same arguments minus the workspace and allocates nothing: its
+ * scratch is a fixed array of GEOCACHE_NOALLOC_MAX_WORKSPACE_FLOATS floats
+ * (16 MiB) in the library's device image, present on every device that loads
+ * the library until the process exits.
+ *  - A step that needs more scratch (geocache_transport_workspace(corr, C)
+ *    larger than the array) is rejected with GEOCACHE_ESHAPE.
+ *  - The first call on each device looks up the array's device address with
+ *    that device current; make that first call before any stream capture.
+ *  - Every call on a device shares the one array, which keeps the previous
+ *    call's contents; nothing in it needs to start at zero (each entry a call
+ *    reads is written earlier in the same call), but calls that overlap on
+ *    the GPU (e.g. on different streams) race and must not be issued.
+ * Returns the statuses of geocache_transport_step.
+ * ------------------------------------------------------------------------ */
+#define GEOCACHE_NOALLOC_MAX_WORKSPACE_FLOATS (4 * 1024 * 1024)
+int geocache_transport_step_noalloc(const geocache_corr* corr, const int32_t* anchors, int a, int C,
+                                    const float* x0_anchor_new, const float* x0_prev, float* x0_out,
+                                    const void* x_t, void* x_next, geocache_dtype lat_dtype,
+                                    const geocache_recon* recon, void* stream);
+
 /* Thread-local description of the last non-OK status of this thread ("" if
  * none).  The pointer stays valid until the thread's next library call. */
 const char* geocache_last_error(void);

@@ -101,6 +101,16 @@ int read_total(const geocache_corr* c, int64_t* total, cudaStream_t s) {
 
 }  // namespace
 
+int geocache::set_error(int status, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return status;
+}
+
 extern "C" {
 
 int geocache_abi_version(void) { return GEOCACHE_ABI_VERSION; }

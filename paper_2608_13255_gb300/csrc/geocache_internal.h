@@ -62,4 +62,7 @@ cudaError_t launch_reconstruct(const void* x_t, const float* x0, void* x_next, i
 
 cudaError_t read_device_error(unsigned int* out, bool clear, cudaStream_t s);
 
+// Records a status and its message for geocache_last_error(); returns status.
+int set_error(int status, const char* fmt, ...);
+
 }  // namespace geocache

@@ -67,7 +67,8 @@ assert ctypes.sizeof(Camera) == 64
 _LIB = None
 EXPORTS = ("geocache_build_corr", "geocache_transport_step", "geocache_reconstruct", "geocache_is_full_step",
            "geocache_rotate_anchors", "geocache_device_status", "geocache_corr_record_count",
-           "geocache_transport_workspace", "geocache_last_error", "geocache_abi_version")
+           "geocache_transport_workspace", "geocache_transport_step_noalloc", "geocache_last_error",
+           "geocache_abi_version")
 
 
 def lib_path() -> str:
@@ -87,6 +88,9 @@ def load():
         L.geocache_build_corr.argtypes = [ctypes.POINTER(Corr), P]
         L.geocache_transport_step.argtypes = [ctypes.POINTER(Corr), P, i, i, P, P, P, P, P, i,
                                               ctypes.POINTER(Recon), P, i64, P]
+        L.geocache_transport_step_noalloc.argtypes = [ctypes.POINTER(Corr), P, i, i, P, P, P, P, P, i,
+                                                      ctypes.POINTER(Recon), P]
+        L.geocache_transport_step_noalloc.restype = ctypes.c_int
         L.geocache_corr_record_count.argtypes = [ctypes.POINTER(Corr), ctypes.POINTER(ctypes.c_int64), P]
         L.geocache_corr_record_count.restype = ctypes.c_int
         L.geocache_transport_workspace.argtypes = [ctypes.POINTER(Corr), i]
@@ -290,6 +294,29 @@ def transport_step(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev, x0_out,
         _dev(workspace, torch.float32, None, "workspace"), 0 if workspace is None else workspace.numel(),
         _stream(stream))
     _check(st)
+
+
+def transport_step_noalloc(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev, x0_out, x_t=None, x_next=None,
+                           recon: Recon | None = None, stream=None):
+    """geocache_transport_step_noalloc: the cached step for callers that
+    cannot supply a workspace (the library's built-in scratch array is used;
+    calls on one device must not overlap on the GPU)."""
+    c = corr.c
+    anc = sorted(int(a) for a in anchors)
+    a = len(anc)
+    n_all = c.B * c.N * C * c.H * c.W
+    arr = (ctypes.c_int32 * max(1, a))(*anc)
+    lat = F32
+    pt = pn = None
+    if recon is not None:
+        lat = _lat_dtype(x_t)
+        pt, pn = _dev(x_t, x_t.dtype, n_all, "x_t"), _dev(x_next, x_t.dtype, n_all, "x_next")
+        _check_pred(recon, n_all)
+    _check(load().geocache_transport_step_noalloc(
+        ctypes.byref(c), ctypes.cast(arr, ctypes.c_void_p), a, int(C),
+        _dev(x0_anchor_new, torch.float32, c.B * a * C * c.H * c.W, "x0_anchor_new"),
+        _dev(x0_prev, torch.float32, n_all, "x0_prev"), _dev(x0_out, torch.float32, n_all, "x0_out"),
+        pt, pn, lat, ctypes.byref(recon) if recon is not None else None, _stream(stream)))
 
 
 def reconstruct(x_t, x0, x_next, recon: Recon, x0_store=None, stream=None):
