@@ -37,7 +37,7 @@ L2_BYTES = 129 * 1024 * 1024
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--steps", type=int, default=200)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="batch128")
@@ -141,8 +141,8 @@ class Trajectory:
                 "anchor": {t: pin(v) for t, v in self.anchor_x0.items()}}
 
     def run(self, events=None):
-        """Enqueue one trajectory; returns the number of kernels launched.
-        events: list receiving (start, end) CUDA events around each cached-step launch."""
+        """Enqueue one trajectory eagerly; returns the number of kernels launched.
+        events: list receiving (start, end) CUDA events around each cached step."""
         import torch
         gc, w = self.gc, self.w
         launches = 0
@@ -152,27 +152,71 @@ class Trajectory:
             launches += 3  # tile counts, their scan, the records
         cache = None
         for t in range(w.S):
-            anchors, full = gc.rotate_anchors(w.N, w.a, t, w.S, self.sched)
-            if full:
-                cache = self.full_x0[t]
-                gc.reconstruct(self.x, cache, self.x, self.recon[t])
-                launches += 1
-            else:
-                out = self.bufs[0] if cache is not self.bufs[0] else self.bufs[1]
-                if events is not None:
-                    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                    e0.record()
-                gc.transport_step(self.corr, anchors, w.C, self.anchor_x0[t], cache, out, self.x, self.x,
-                                  self.recon[t], workspace=self.workspace)
-                if events is not None:
-                    e1.record()
-                    events.append((e0, e1))
-                launches += gc.transport_launches(w.a, w.N, self.corr.c.mode, in_place=False)
-                cache = out
+            timed = events is not None and t in self.anchor_x0
+            if timed:
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+            cache, n = self._step(t, cache)
+            launches += n
+            if timed:
+                e1.record()
+                events.append((e0, e1))
+        self.launches = launches
         return launches
 
-    def run_e2e(self, host):
-        """One trajectory from pinned host inputs to a host copy of the final latents."""
+    def _step(self, t, cache):
+        """Enqueue sampler step t; returns (new cache, kernels launched)."""
+        gc, w = self.gc, self.w
+        anchors, full = gc.rotate_anchors(w.N, w.a, t, w.S, self.sched)
+        if full:
+            gc.reconstruct(self.x, self.full_x0[t], self.x, self.recon[t])
+            return self.full_x0[t], 1
+        out = self.bufs[0] if cache is not self.bufs[0] else self.bufs[1]
+        gc.transport_step(self.corr, anchors, w.C, self.anchor_x0[t], cache, out, self.x, self.x, self.recon[t],
+                          workspace=self.workspace)
+        return out, gc.transport_launches(w.a, w.N, self.corr.c.mode, in_place=False)
+
+    def capture(self):
+        """Capture the correspondence build and every sampler step in CUDA
+        graphs; False (and eager launches) if capture is unavailable."""
+        import torch
+        self.run()  # lazy initialisation outside capture
+        torch.cuda.synchronize()
+        try:
+            self.g_build = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(self.g_build):
+                self.gc.build_corr(self.corr)
+            self.g_steps = []
+            cache = None
+            for t in range(self.w.S):
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    cache, _ = self._step(t, cache)
+                self.g_steps.append(g)
+            self.replay(None)
+            torch.cuda.synchronize()
+            return True
+        except RuntimeError as exc:
+            print("bench: CUDA graph capture failed (%s); timing eager launches" % exc, file=sys.stderr)
+            self.g_build = self.g_steps = None
+            return False
+
+    def replay(self, events=None):
+        import torch
+        self.g_build.replay()
+        for t, g in enumerate(self.g_steps):
+            timed = events is not None and t in self.anchor_x0
+            if timed:
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+            g.replay()
+            if timed:
+                e1.record()
+                events.append((e0, e1))
+
+    def run_e2e(self, host, graph=None):
+        """One trajectory from pinned host inputs to a host copy of the final
+        latents (the trajectory itself replayed from `graph` when given)."""
         import torch
         self.pos.copy_(host["pos"], non_blocking=True)
         self.valid.copy_(host["valid"], non_blocking=True)
@@ -182,7 +226,10 @@ class Trajectory:
             self.full_x0[t].copy_(v, non_blocking=True)
         for t, v in host["anchor"].items():
             self.anchor_x0[t].copy_(v, non_blocking=True)
-        self.run()
+        if graph:
+            self.replay()
+        else:
+            self.run()
         out = torch.empty(self.x.shape, dtype=self.x.dtype, pin_memory=True)
         out.copy_(self.x, non_blocking=True)
         torch.cuda.current_stream().synchronize()
@@ -214,7 +261,7 @@ class ClockSampler:
             os.makedirs(os.path.dirname(self.path), exist_ok=True)
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.FIELDS,
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=self.f, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
@@ -343,16 +390,30 @@ def main():
     traj = Trajectory(w, dev, args.corr)
     ws_bytes = traj.working_set()
 
-    args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
-    for _ in range(args.warmup):
-        traj.run()
-    torch.cuda.synchronize()
-
     def barrier():
         if world > 1:
             dist.barrier()
 
+    # every kernel launch of a trajectory is captured once in CUDA graphs (one
+    # for the correspondence build, one per sampler step) and replayed, so
+    # launches cost no host time; events between the replays time each
+    # cached step's transport kernels
     events = []
+    use_graphs = traj.capture()
+    launches_per_traj = traj.launches
+
+    def one_step(ev=None):
+        if use_graphs:
+            traj.replay(ev)
+        else:
+            traj.run(ev)
+        return launches_per_traj
+
+    args.warmup = max(3, args.warmup)  # at least three untimed warm-up steps
+    for _ in range(args.warmup):
+        one_step()
+    torch.cuda.synchronize()
+
     launches = 0
     with ClockSampler(local) as clocks:
         barrier()
@@ -361,7 +422,7 @@ def main():
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record()
         for _ in range(args.steps):
-            launches += traj.run(events)
+            launches += one_step(events)
         t1.record()
         torch.cuda.synchronize()
         barrier()
@@ -392,11 +453,11 @@ def main():
     e2e = None
     if not args.no_e2e:
         host = traj.host_inputs()
-        traj.run_e2e(host)
+        traj.run_e2e(host, use_graphs)
         barrier()
         t_s = time.perf_counter()
         for _ in range(args.steps):
-            out = traj.run_e2e(host)
+            out = traj.run_e2e(host, use_graphs)
         e2e_s = (time.perf_counter() - t_s) / args.steps
         if world > 1:
             tt = torch.tensor([e2e_s], dtype=torch.float64)
@@ -415,8 +476,9 @@ def main():
                    "storage": "bf16 latents, f32 x0 cache" if w.dtype == "bf16" else "f32",
                    "l2": "inputs larger than L2: %.0f MB touched per cached step vs %d MB L2" % (
                        ws_bytes / 1e6, L2_BYTES // 2 ** 20),
-                   "step": "tau + %d-step trajectory (%d cached transport steps, %d full steps)" % (
-                       w.S, traj.n_cached, w.S - traj.n_cached)},
+                   "step": "tau + correspondence build + %d-step trajectory (%d cached transport steps, %d full "
+                           "steps)" % (w.S, traj.n_cached, w.S - traj.n_cached),
+                   "launch": "CUDA graphs (one per sampler step) replayed" if use_graphs else "eager"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
                      "kernel": "transport_kernel", "alg_bytes_per_launch": alg,

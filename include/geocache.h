@@ -8,8 +8,9 @@
  * - Pointers marked "device" are CUDA device addresses on the current device
  *   (e.g. torch tensors' data_ptr()); pointers marked "host" are ordinary host
  *   memory.  The caller owns every buffer and the library allocates no
- *   memory; its only device-resident state is a 4-byte status word that
- *   kernels set when a bounded wait gives up (geocache_device_status).
+ *   memory; its device-resident state is a 4-byte status word that kernels
+ *   set on a failure they can only detect on the GPU (geocache_device_status)
+ *   and the fixed scratch array of geocache_transport_step_noalloc.
  * - Every device-side entry point is asynchronous on `stream` (a cudaStream_t,
  *   NULL = the legacy default stream) and returns after enqueueing its kernels.
  * - Latents are NCHW per view with the views on the batch axis:
@@ -161,9 +162,10 @@ typedef struct {
  * the keep masks (when keep is non-NULL): the diagonal u == v and
  * background targets hold idx -1 / w 0 / keep 0.  When tile_ptr is given
  * (it needs keep) the tile offsets of the sparse form are written, and when
- * records is also given the records are written; this last part reads the
- * record count back to the host (the call then synchronises `stream`) and
- * fails with ESHAPE if it exceeds max_records (see geocache_corr_record_count).
+ * records is also given the records are written.  The call is asynchronous;
+ * size records with geocache_corr_record_count (the count depends only on
+ * the geometry).  Records beyond max_records are dropped and flagged in the
+ * device status word (geocache_device_status then returns ESHAPE).
  * Sizes: 1 <= B, 2 <= N <= GEOCACHE_MAX_VIEWS, 1 <= H, W <= 16384,
  * K in {1, 4}, 0 < tol_frac.  Outputs must not overlap the inputs.
  * Returns GEOCACHE_OK, EINVAL (NULL / bad K / tol_frac), ESHAPE, EALIAS, ECUDA.
@@ -261,11 +263,12 @@ int geocache_rotate_anchors(int N, int a, int step, int S, const geocache_schedu
 
 /* --------------------------------------------------------------------------
  * geocache_device_status -- synchronises `stream`, then reads and clears the
- * device status word.  Every wait inside the kernels (the completion of their
- * own bulk copies into shared memory) is bounded in time; a CTA whose wait
- * runs out sets the word and returns without writing its outputs, so the
- * context stays usable.  Returns GEOCACHE_OK, ETIMEOUT (some call since the
- * last check left outputs incomplete) or ECUDA.
+ * device status word.  Failures only the GPU can see set it instead of
+ * trapping, so the context stays usable: a sparse-form build whose records
+ * exceed max_records (the excess is dropped; transport steps read only the
+ * records that exist), and a bounded wait inside a kernel that ran out (its
+ * CTA returns without writing its outputs).  Returns GEOCACHE_OK, ESHAPE
+ * (record overflow), ETIMEOUT (a wait gave up) or ECUDA.
  * ------------------------------------------------------------------------ */
 int geocache_device_status(void* stream);
 

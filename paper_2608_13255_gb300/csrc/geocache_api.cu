@@ -119,6 +119,9 @@ int geocache_device_status(void* stream) {
     unsigned int word = 0;
     cudaError_t e = geocache::read_device_error(&word, true, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "reading the device status word");
+    if (word & 2u)
+        return fail(GEOCACHE_ESHAPE, "a sparse-form build had more records than max_records (status word 0x%x); "
+                                     "query geocache_corr_record_count and rebuild", word);
     if (word) return fail(GEOCACHE_ETIMEOUT, "a bounded device wait gave up (status word 0x%x); outputs of that call are incomplete", word);
     return ok();
 }
@@ -175,12 +178,6 @@ int geocache_build_corr(geocache_corr* c, void* stream) {
         if (e != cudaSuccess) return cuda_fail(e, "tile-offset kernel launch");
     }
     if (c->records) {
-        int64_t total = 0;
-        st = read_total(c, &total, s);
-        if (st) return st;
-        if (total > c->max_records)
-            return fail(GEOCACHE_ESHAPE, "the sparse form has %lld records but max_records is %lld",
-                        (long long)total, (long long)c->max_records);
         e = geocache::launch_fill_records(*c, s);
         if (e != cudaSuccess) return cuda_fail(e, "record kernel launch");
     }
@@ -279,6 +276,7 @@ int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int 
     t.keep = c->keep;
     t.tile_ptr = c->tile_ptr;
     t.records = c->records;
+    t.max_records = c->max_records;
     t.workspace = workspace;
     t.x0_new = x0_anchor_new; t.x0_prev = x0_prev; t.x0_out = x0_out;
     t.x_t = x_t; t.x_next = x_next; t.pred_out = recon ? recon->pred_out : nullptr;

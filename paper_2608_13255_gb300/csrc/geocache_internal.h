@@ -34,6 +34,7 @@ struct TransportArgs {
     const uint8_t* keep;
     const int32_t* tile_ptr;
     const geocache_tap_record* records;
+    long long max_records;
     float* workspace;
     const float* x0_new;
     const float* x0_prev;

@@ -165,6 +165,11 @@ cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+// Device status word (the library's only device-resident state): bit 0 = a
+// bounded wait gave up, bit 1 = the sparse form did not fit max_records.
+// Read and cleared by geocache_device_status().
+__device__ unsigned int g_device_error = 0;
+
 // ---------------------------------------------------- sparse operator --
 // G_{u->v} in tile-CSR form: for each (asset b, target view v, source view u,
 // tile of GEOCACHE_TILE_TOKENS tokens) the records of its kept rows, in token
@@ -309,7 +314,10 @@ __global__ void __launch_bounds__(256) fill_records_kernel(const float* __restri
         out.q_tl = f.j0 * W + f.i0;
         out.fx = K == 4 ? f.ax[1] : 0.0f;
         out.fy = K == 4 ? f.ay[1] : 0.0f;
-        if (r < max_records) reinterpret_cast<int4*>(rec)[r] = *reinterpret_cast<const int4*>(&out);
+        if (r < max_records)
+            reinterpret_cast<int4*>(rec)[r] = *reinterpret_cast<const int4*>(&out);
+        else
+            atomicOr(&g_device_error, 2u);  // records beyond the capacity are dropped
         ++r;
     }
 }
@@ -464,10 +472,6 @@ constexpr int kChunk = 4;                        // anchors per work-list round
 constexpr int kPairCap = kChunk * kTileTokens;   // (token, anchor) work items of one round
 constexpr int kStages = 2;
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // bounded mbarrier wait: 2 s
-
-// Device error word (the library's only device-resident state): bit 0 is set
-// when a bounded wait gave up.  Read and cleared by geocache_device_status().
-__device__ unsigned int g_device_error = 0;
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
@@ -1003,7 +1007,9 @@ __device__ __forceinline__ void apply_records(const TransportArgs& args, int pai
     const int v = nonanchor_view(args, vi);
     const int u = args.anchors[s2];
     const size_t pair = ((size_t)b * N + v) * N + u;
-    const int r0 = __ldg(args.tile_ptr + pair * T), r1 = __ldg(args.tile_ptr + pair * T + T);
+    const long long cap = args.max_records;
+    const int r0 = (int)min((long long)__ldg(args.tile_ptr + pair * T), cap);
+    const int r1 = (int)min((long long)__ldg(args.tile_ptr + pair * T + T), cap);
     const size_t plane = (size_t)HW;
     const float* xn = args.x0_new + ((size_t)b * a + s2) * C * plane;
     const float* xp = args.x0_prev + ((size_t)b * N + u) * C * plane;
@@ -1115,9 +1121,10 @@ __global__ void __launch_bounds__(kThreads) sparse_phase_b_kernel(const Transpor
     if (cnt > 0) q.load(args, b, v, -1, p0, cnt, 0, C < 4 ? C : 4);
     if (t < a) {
         const size_t i = (((size_t)b * N + v) * N + args.anchors[t]) * T_tiles + tile;
-        const int r0 = __ldg(args.tile_ptr + i);
+        // ranges clamped to the records that exist (an overflow is reported by the build)
+        const int r0 = (int)min((long long)__ldg(args.tile_ptr + i), args.max_records);
         s_r0[t] = r0;
-        s_cnt[t] = __ldg(args.tile_ptr + i + 1) - r0;
+        s_cnt[t] = (int)min((long long)__ldg(args.tile_ptr + i + 1), args.max_records) - r0;
     }
     pdl_wait();  // phase A's workspace writes are complete and visible
     __syncthreads();

@@ -356,3 +356,50 @@ def test_trajectory_per_step_parity_and_drift(gc, workloads):
     drift = np.abs(x.cpu().float().numpy().astype(np.float64) - x_or).max()
     print("end-of-trajectory drift (GPU vs oracle's own trajectory): %.4g" % drift)
     assert drift < 0.25
+
+
+def test_record_overflow_is_reported_not_faulted(gc, workloads):
+    # a sparse form built into too few records: the excess is dropped and
+    # flagged in the device status word; a transport step over it reads only
+    # the records that exist (no fault), and the status is reported
+    w = workloads("hunyuan64")
+    g = DeviceGeometry(w, K=4, tables=False)
+    short = torch.empty((g.n_records // 2, 4), dtype=torch.int32, device="cuda")
+    c = gc.make_corr(g.pos, g.valid, g.cams, g.tau, K=4, keep=g.keep, tile_ptr=g.tile_ptr, records=short,
+                     mode=gc.CORR_SPARSE)
+    gc.build_corr(c)
+    with pytest.raises(gc.GeocacheError) as ei:
+        gc.device_status()
+    assert ei.value.status == gc.ESHAPE
+    gc.device_status()  # cleared by the read
+    x0_prev, x0_new, _ = step_inputs(w, 3, [0, 3])
+    d_prev, d_new = torch.from_numpy(x0_prev).cuda(), torch.from_numpy(x0_new).cuda()
+    out = torch.empty_like(d_prev)
+    ws = torch.empty(max(c.workspace_floats(w.C), 4), device="cuda")
+    gc.transport_step(c, [0, 3], w.C, d_new, d_prev, out, workspace=ws)
+    torch.cuda.synchronize()
+    gc.device_status()
+    assert torch.isfinite(out).all()
+
+
+def test_graph_replay_matches_eager(gc, workloads):
+    # a cached step captured in a CUDA graph (with the programmatic
+    # dependency between its two kernels) gives the eager results
+    w = workloads("batch128")
+    g = DeviceGeometry(w, K=4, tables=False)
+    x0_prev, x0_new, xt32 = step_inputs(w, 5, [1, 4])
+    _, xt = latent_values(xt32, w)
+    d_prev, d_new, d_xt = torch.from_numpy(x0_prev).cuda(), torch.from_numpy(x0_new).cuda(), xt.cuda()
+    ws = g.workspace(w.C)
+    p = synth.recon_params(w, 5)
+    r = gc.make_recon("ddim", a_t=p["a_t"], a_prev=p["a_prev"])
+    out_e, xn_e = torch.empty_like(d_prev), torch.empty_like(d_xt)
+    gc.transport_step(g.corr, [1, 4], w.C, d_new, d_prev, out_e, d_xt, xn_e, r, workspace=ws)
+    out_g, xn_g = torch.empty_like(d_prev), torch.empty_like(d_xt)
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        gc.transport_step(g.corr, [1, 4], w.C, d_new, d_prev, out_g, d_xt, xn_g, r, workspace=ws)
+    graph.replay()
+    torch.cuda.synchronize()
+    assert torch.equal(out_g, out_e)
+    assert torch.equal(xn_g.view(torch.int16), xn_e.view(torch.int16))
