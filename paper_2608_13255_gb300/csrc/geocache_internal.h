@@ -54,7 +54,7 @@ cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s);
 // tile_ptr (tile_ptr[n] = total, or -1 when the total exceeds INT32_MAX)
 cudaError_t launch_tile_ptr(const geocache_corr& c, cudaStream_t s);
 cudaError_t launch_fill_records(const geocache_corr& c, cudaStream_t s);
-int tiles_per_view(int H, int W);
+__host__ __device__ int tiles_per_view(int H, int W);
 cudaError_t launch_transport(const TransportArgs& t, cudaStream_t s);
 int transport_launch_count(int a, int C, int in_place);
 cudaError_t launch_copy_anchor_rows(const TransportArgs& t, cudaStream_t s);

@@ -4,6 +4,8 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <cooperative_groups.h>
+
 #include <cfloat>
 #include <cstdint>
 
@@ -11,6 +13,8 @@
 #include "geocache_internal.h"
 
 namespace geocache {
+
+__host__ __device__ int tiles_per_view(int H, int W) { return (H * W + GEOCACHE_TILE_TOKENS - 1) / GEOCACHE_TILE_TOKENS; }
 
 // ---------------------------------------------------------------- latents --
 __device__ __forceinline__ float lat_load(const float* p, size_t i) { return __ldg(p + i); }
@@ -38,130 +42,184 @@ __device__ __forceinline__ float recon_one(const ReconCoef& c, float xt, float x
 }
 
 // -------------------------------------------------------------------- tau --
-// One CTA per asset: componentwise min / max of the foreground texels of all
-// N views (order-free and exact), then tau = tol_frac * sqrt(diag^2) with the
-// squares summed ((d0^2 + d1^2) + d2^2) in binary32.
-__global__ void __launch_bounds__(1024) tau_kernel(const float* __restrict__ pos,
-                                                   const uint8_t* __restrict__ valid, int N, int H,
-                                                   int W, float tol_frac, float* __restrict__ tau) {
-    const int b = blockIdx.x;
-    const size_t per = (size_t)N * H * W;
-    const float* P = pos + 3 * per * b;
-    const uint8_t* V = valid + per * b;
-    float lo[3] = {FLT_MAX, FLT_MAX, FLT_MAX}, hi[3] = {-FLT_MAX, -FLT_MAX, -FLT_MAX};
-    int any = 0;
-    for (size_t i = threadIdx.x; i < per; i += blockDim.x) {
-        if (!V[i]) continue;
-        any = 1;
-#pragma unroll
-        for (int c = 0; c < 3; ++c) {
-            const float x = P[3 * i + c];
-            lo[c] = fminf(lo[c], x);
-            hi[c] = fmaxf(hi[c], x);
-        }
-    }
+// One thread-block cluster per asset: CTA r of the cluster reduces the
+// componentwise min / max of the foreground texels of views r, r + CS, ...
+// (exact and order-free), the cluster combines the partial boxes through
+// distributed shared memory, and CTA 0 writes tau = tol_frac * sqrt(diag^2)
+// with the squares summed ((d0^2 + d1^2) + d2^2) in binary32.
+struct Box {
+    float lo[3], hi[3];
+    int any;
+};
+
+__device__ __forceinline__ void box_reduce_warp(Box& x) {
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
 #pragma unroll
         for (int c = 0; c < 3; ++c) {
-            lo[c] = fminf(lo[c], __shfl_xor_sync(0xffffffffu, lo[c], off));
-            hi[c] = fmaxf(hi[c], __shfl_xor_sync(0xffffffffu, hi[c], off));
+            x.lo[c] = fminf(x.lo[c], __shfl_xor_sync(0xffffffffu, x.lo[c], off));
+            x.hi[c] = fmaxf(x.hi[c], __shfl_xor_sync(0xffffffffu, x.hi[c], off));
         }
-        any |= __shfl_xor_sync(0xffffffffu, any, off);
+        x.any |= __shfl_xor_sync(0xffffffffu, x.any, off);
     }
-    __shared__ float s_lo[32][3], s_hi[32][3];
-    __shared__ int s_any[32];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) {
+}
+
+__global__ void __launch_bounds__(512) tau_kernel(const float* __restrict__ pos, const uint8_t* __restrict__ valid,
+                                                  int N, int HW, float tol_frac, float* __restrict__ tau) {
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    const int cs = (int)cluster.num_blocks();
+    const int rank = (int)cluster.block_rank();
+    const int b = blockIdx.x / cs;
+    __shared__ Box s_warp[16];
+    __shared__ Box s_part;
+    Box x;
 #pragma unroll
-        for (int c = 0; c < 3; ++c) { s_lo[warp][c] = lo[c]; s_hi[warp][c] = hi[c]; }
-        s_any[warp] = any;
+    for (int c = 0; c < 3; ++c) { x.lo[c] = FLT_MAX; x.hi[c] = -FLT_MAX; }
+    x.any = 0;
+    for (int v = rank; v < N; v += cs) {
+        const size_t base = ((size_t)b * N + v) * HW;
+        for (int i = threadIdx.x; i < HW; i += blockDim.x) {
+            if (!__ldg(valid + base + i)) continue;
+            x.any = 1;
+#pragma unroll
+            for (int c = 0; c < 3; ++c) {
+                const float p = __ldg(pos + 3 * (base + i) + c);
+                x.lo[c] = fminf(x.lo[c], p);
+                x.hi[c] = fmaxf(x.hi[c], p);
+            }
+        }
     }
+    box_reduce_warp(x);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) s_warp[warp] = x;
     __syncthreads();
     if (warp == 0) {
         const int nw = blockDim.x >> 5;
+        if (lane < nw) x = s_warp[lane];
+        else {
 #pragma unroll
-        for (int c = 0; c < 3; ++c) {
-            lo[c] = lane < nw ? s_lo[lane][c] : FLT_MAX;
-            hi[c] = lane < nw ? s_hi[lane][c] : -FLT_MAX;
+            for (int c = 0; c < 3; ++c) { x.lo[c] = FLT_MAX; x.hi[c] = -FLT_MAX; }
+            x.any = 0;
         }
-        any = lane < nw ? s_any[lane] : 0;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) {
+        box_reduce_warp(x);
+        if (lane == 0) s_part = x;
+    }
+    cluster.sync();  // every CTA's partial box is in its shared memory
+    if (rank == 0 && threadIdx.x == 0) {
+        Box t = s_part;
+        for (int r = 1; r < cs; ++r) {
+            const Box* o = cluster.map_shared_rank(&s_part, r);
 #pragma unroll
             for (int c = 0; c < 3; ++c) {
-                lo[c] = fminf(lo[c], __shfl_xor_sync(0xffffffffu, lo[c], off));
-                hi[c] = fmaxf(hi[c], __shfl_xor_sync(0xffffffffu, hi[c], off));
+                t.lo[c] = fminf(t.lo[c], o->lo[c]);
+                t.hi[c] = fmaxf(t.hi[c], o->hi[c]);
             }
-            any |= __shfl_xor_sync(0xffffffffu, any, off);
+            t.any |= o->any;
         }
-        if (lane == 0) {
-            float t = 0.0f;
-            if (any) {
-                const float d0 = __fsub_rn(hi[0], lo[0]), d1 = __fsub_rn(hi[1], lo[1]),
-                            d2 = __fsub_rn(hi[2], lo[2]);
-                const float diag2 =
-                    __fadd_rn(__fadd_rn(__fmul_rn(d0, d0), __fmul_rn(d1, d1)), __fmul_rn(d2, d2));
-                t = __fmul_rn(tol_frac, __fsqrt_rn(diag2));
-            }
-            tau[b] = t;
+        float tv = 0.0f;
+        if (t.any) {
+            const float d0 = __fsub_rn(t.hi[0], t.lo[0]), d1 = __fsub_rn(t.hi[1], t.lo[1]),
+                        d2 = __fsub_rn(t.hi[2], t.lo[2]);
+            const float diag2 = __fadd_rn(__fadd_rn(__fmul_rn(d0, d0), __fmul_rn(d1, d1)), __fmul_rn(d2, d2));
+            tv = __fmul_rn(tol_frac, __fsqrt_rn(diag2));
         }
+        tau[b] = tv;
     }
+    cluster.sync();  // the other CTAs' shared memory stays alive until CTA 0 has read it
 }
 
 cudaError_t launch_tau(const float* pos, const uint8_t* valid, int B, int N, int H, int W, float tol_frac,
                        float* tau, cudaStream_t s) {
-    tau_kernel<<<B, 1024, 0, s>>>(pos, valid, N, H, W, tol_frac, tau);
-    return cudaGetLastError();
+    const int cs = N < 8 ? N : 8;  // portable cluster size
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(B * cs);
+    cfg.blockDim = dim3(512);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, tau_kernel, pos, valid, N, H * W, tol_frac, tau);
 }
 
 // ------------------------------------------------------- correspondence --
-// One thread per (asset b, target view v, source view u, token p): the
-// tables idx/w (when non-NULL) and the keep masks (when non-NULL).
+// One thread per (asset b, target view v, token p), looping over the source
+// views u: the target's position is loaded once.  Writes the keep masks and
+// (when requested) the idx/w tables of every pair; with tile_cnt given, adds
+// the kept rows of each (b, v, u, tile) to its count (one atomic per warp:
+// a warp's 32 tokens lie in one tile).
 template <int K>
 __global__ void __launch_bounds__(256) build_corr_kernel(const float* __restrict__ pos,
                                                          const uint8_t* __restrict__ valid,
                                                          const geocache_camera* __restrict__ cams,
                                                          const float* __restrict__ tau, int N, int H, int W,
                                                          int32_t* __restrict__ idx, float* __restrict__ wout,
-                                                         uint8_t* __restrict__ keep) {
+                                                         uint8_t* __restrict__ keep, int32_t* __restrict__ tile_cnt) {
     const int HW = H * W;
     const int p = blockIdx.x * blockDim.x + threadIdx.x;
-    const int v = blockIdx.y / N, u = blockIdx.y % N, b = blockIdx.z;
-    __shared__ geocache_camera s_cam;
-    if (threadIdx.x < 16) reinterpret_cast<float*>(&s_cam)[threadIdx.x] =
-        __ldg(reinterpret_cast<const float*>(cams + (size_t)b * N + u) + threadIdx.x);
+    const int v = blockIdx.y, b = blockIdx.z;
+    __shared__ geocache_camera s_cam[GEOCACHE_MAX_VIEWS];
+    for (int i = threadIdx.x; i < N * 16; i += blockDim.x)
+        reinterpret_cast<float*>(s_cam)[i] = __ldg(reinterpret_cast<const float*>(cams + (size_t)b * N) + i);
     __syncthreads();
-    if (p >= HW) return;
-    Taps t;
-    taps_clear(t);
-    int mask = 0;
-    const size_t tv = ((size_t)b * N + v) * HW + p;
-    if (u != v && __ldg(valid + tv)) {
+    const bool in = p < HW;
+    const size_t tv = ((size_t)b * N + v) * HW + (in ? p : 0);
+    const bool fg = in && __ldg(valid + tv);
+    float X0 = 0.f, X1 = 0.f, X2 = 0.f, tau2 = 0.f;
+    if (fg) {
+        X0 = __ldg(pos + 3 * tv);
+        X1 = __ldg(pos + 3 * tv + 1);
+        X2 = __ldg(pos + 3 * tv + 2);
         const float tu = __ldg(tau + b);
-        const size_t su = ((size_t)b * N + u) * HW;
-        compute_taps<K>(s_cam, pos + 3 * su, valid + su, H, W, __ldg(pos + 3 * tv), __ldg(pos + 3 * tv + 1),
-                        __ldg(pos + 3 * tv + 2), __fmul_rn(tu, tu), t, &mask);
+        tau2 = __fmul_rn(tu, tu);
     }
-    const size_t row = (((size_t)b * N + v) * N + u) * HW + p;
-    if (keep) keep[row] = (uint8_t)mask;
-    if (!idx) return;
-    if (K == 4) {
-        reinterpret_cast<int4*>(idx)[row] = make_int4(t.q[0], t.q[1], t.q[2], t.q[3]);
-        reinterpret_cast<float4*>(wout)[row] = make_float4(t.w[0], t.w[1], t.w[2], t.w[3]);
-    } else {
-        idx[row] = t.q[0];
-        wout[row] = t.w[0];
+    const int T = tiles_per_view(H, W);
+    for (int u = 0; u < N; ++u) {
+        Taps t;
+        taps_clear(t);
+        int mask = 0;
+        if (fg && u != v) {
+            const size_t su = ((size_t)b * N + u) * HW;
+            compute_taps<K>(s_cam[u], pos + 3 * su, valid + su, H, W, X0, X1, X2, tau2, t, &mask);
+        }
+        if (tile_cnt) {
+            const unsigned kept = __ballot_sync(0xffffffffu, mask != 0);
+            if ((threadIdx.x & 31) == 0 && kept)
+                atomicAdd(tile_cnt + (((size_t)b * N + v) * N + u) * T + (blockIdx.x * blockDim.x) / GEOCACHE_TILE_TOKENS,
+                          __popc(kept));
+        }
+        if (!in) continue;
+        const size_t row = (((size_t)b * N + v) * N + u) * HW + p;
+        if (keep) keep[row] = (uint8_t)mask;
+        if (!idx) continue;
+        if (K == 4) {
+            reinterpret_cast<int4*>(idx)[row] = make_int4(t.q[0], t.q[1], t.q[2], t.q[3]);
+            reinterpret_cast<float4*>(wout)[row] = make_float4(t.w[0], t.w[1], t.w[2], t.w[3]);
+        } else {
+            idx[row] = t.q[0];
+            wout[row] = t.w[0];
+        }
     }
 }
 
 cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s) {
     const int HW = c.H * c.W;
-    dim3 grid((HW + 255) / 256, c.N * c.N, c.B);
+    dim3 grid((HW + 255) / 256, c.N, c.B);
+    int32_t* cnt = nullptr;
+    if (c.tile_ptr) {
+        const size_t n = (size_t)c.B * c.N * c.N * tiles_per_view(c.H, c.W) + 1;
+        cudaError_t e = cudaMemsetAsync(c.tile_ptr, 0, n * sizeof(int32_t), s);
+        if (e != cudaSuccess) return e;
+        cnt = c.tile_ptr;
+    }
     if (c.K == 4)
-        build_corr_kernel<4><<<grid, 256, 0, s>>>(c.pos, c.valid, c.cams, c.tau, c.N, c.H, c.W, c.idx, c.w, c.keep);
+        build_corr_kernel<4><<<grid, 256, 0, s>>>(c.pos, c.valid, c.cams, c.tau, c.N, c.H, c.W, c.idx, c.w, c.keep, cnt);
     else
-        build_corr_kernel<1><<<grid, 256, 0, s>>>(c.pos, c.valid, c.cams, c.tau, c.N, c.H, c.W, c.idx, c.w, c.keep);
+        build_corr_kernel<1><<<grid, 256, 0, s>>>(c.pos, c.valid, c.cams, c.tau, c.N, c.H, c.W, c.idx, c.w, c.keep, cnt);
     return cudaGetLastError();
 }
 
@@ -174,31 +232,8 @@ __device__ unsigned int g_device_error = 0;
 // G_{u->v} in tile-CSR form: for each (asset b, target view v, source view u,
 // tile of GEOCACHE_TILE_TOKENS tokens) the records of its kept rows, in token
 // order; tile_ptr holds the exclusive prefix sum of the per-tile counts.
-int tiles_per_view(int H, int W) { return (H * W + GEOCACHE_TILE_TOKENS - 1) / GEOCACHE_TILE_TOKENS; }
 __device__ __forceinline__ int tiles_per_view_dev(int H, int W) {
     return (H * W + GEOCACHE_TILE_TOKENS - 1) / GEOCACHE_TILE_TOKENS;
-}
-
-// count of kept rows (non-zero keep bytes) of each (b, v, u, tile)
-__global__ void __launch_bounds__(256) tile_count_kernel(const uint8_t* __restrict__ keep, int N, int HW, int T,
-                                                         int32_t* __restrict__ cnt) {
-    const int tile = blockIdx.x, vu = blockIdx.y, b = blockIdx.z;
-    const uint8_t* row = keep + ((size_t)b * N * N + vu) * HW;
-    const int tile0 = tile * GEOCACHE_TILE_TOKENS;
-    int c = 0;
-    for (int i = threadIdx.x; i < GEOCACHE_TILE_TOKENS; i += blockDim.x) {
-        const int p = tile0 + i;
-        if (p < HW && __ldg(row + p)) ++c;
-    }
-    c = __reduce_add_sync(0xffffffffu, c);
-    __shared__ int s[8];
-    if ((threadIdx.x & 31) == 0) s[threadIdx.x >> 5] = c;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        int tot = 0;
-        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) tot += s[w];
-        cnt[((size_t)b * N * N + vu) * T + tile] = tot;
-    }
 }
 
 // in-place exclusive prefix sum of n counts by one CTA; a[n] = total, or -1
@@ -251,12 +286,10 @@ __global__ void __launch_bounds__(1024) exclusive_scan_kernel(int32_t* a, long l
     if (t == 0) a[n] = s_carry > 0x7fffffffLL ? -1 : (int32_t)s_carry;
 }
 
+// tile_ptr holds the per-tile counts written by build_corr_kernel; turn them
+// into offsets
 cudaError_t launch_tile_ptr(const geocache_corr& c, cudaStream_t s) {
-    const int HW = c.H * c.W, T = tiles_per_view(c.H, c.W);
-    dim3 grid(T, c.N * c.N, c.B);
-    tile_count_kernel<<<grid, 256, 0, s>>>(c.keep, c.N, HW, T, c.tile_ptr);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+    const int T = tiles_per_view(c.H, c.W);
     exclusive_scan_kernel<<<1, 1024, 0, s>>>(c.tile_ptr, (long long)c.B * c.N * c.N * T);
     return cudaGetLastError();
 }
