@@ -50,6 +50,23 @@ def parse():
 
 
 # ------------------------------------------------------------------ setup --
+def reduce_max(x: float, world: int) -> float:
+    """Maximum of a float over all ranks (gloo; no collective on the data path)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_value(pixels_per_rank: float, world: int, seconds: float) -> float:
+    """Whole-job throughput: every rank processes its own assets (weak
+    scaling), the job takes as long as the slowest rank."""
+    return pixels_per_rank * world / seconds
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))
@@ -439,15 +456,11 @@ def main():
         t1.record()
         torch.cuda.synchronize()
         barrier()
-    ms = t0.elapsed_time(t1)
+    ms = reduce_max(t0.elapsed_time(t1), world)
     kernel_ms = [a.elapsed_time(b) for a, b in events]
-    if world > 1:
-        tt = torch.tensor([ms], dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
     ms_per_step = ms / args.steps
     total_pixels = traj.pixels * world
-    value = total_pixels / (ms_per_step / 1e3)
+    value = job_value(traj.pixels, world, ms_per_step / 1e3)
 
     k_avg_ms = sum(kernel_ms) / len(kernel_ms)
     alg = step_bytes(w)
@@ -463,12 +476,8 @@ def main():
         t_s = time.perf_counter()
         for _ in range(args.steps):
             out = traj.run_e2e(host, use_graphs)
-        e2e_s = (time.perf_counter() - t_s) / args.steps
-        if world > 1:
-            tt = torch.tensor([e2e_s], dtype=torch.float64)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e2e_s = float(tt.item())
-        e2e = {"value": total_pixels / e2e_s, "unit": UNIT, "h2d_bytes_per_step": traj.h2d_bytes(),
+        e2e_s = reduce_max((time.perf_counter() - t_s) / args.steps, world)
+        e2e = {"value": job_value(traj.pixels, world, e2e_s), "unit": UNIT, "h2d_bytes_per_step": traj.h2d_bytes(),
                "d2h_bytes_per_step": out.numel() * out.element_size(), "ms_per_step": 1e3 * e2e_s}
 
     if rank != 0:
