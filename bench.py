@@ -147,6 +147,7 @@ class Trajectory:
                 self.anchor_x0[t] = (x0_d[:, anchors] + d).contiguous()
         self.bufs = [torch.empty_like(x0_d), torch.empty_like(x0_d)]
         self.n_cached = len(self.anchor_x0)
+        self.anchor_sets = {tuple(gc.rotate_anchors(w.N, w.a, t, w.S, self.sched)[0]) for t in self.anchor_x0}
         self.pixels = self.n_cached * w.B * (w.N - w.a) * w.H * w.W
 
     def host_inputs(self):
@@ -468,6 +469,41 @@ def main():
     peak, peak_src = measured_peak()
     traffic = measured_traffic(gbuild.source_hash(), w.B)
 
+    # secondary: anchor-row pack of the latents and scatter back (the batch
+    # slicing around the denoiser's anchor-only forward); four source / slice
+    # pairs in rotation (267 MB per cycle, larger than L2) so that each call
+    # reads from HBM; bytes = rows read + rows written
+    pack = None
+    if rank == 0:
+        anchors0 = sorted(next(iter(traj.anchor_sets)))
+        srcs = [traj.x.clone() for _ in range(4)]
+        sls = [torch.empty((w.B, len(anchors0)) + tuple(traj.x.shape[2:]), dtype=traj.x.dtype, device=dev)
+               for _ in range(4)]
+        reps = 48
+        for i in range(4):
+            traj.gc.pack_anchors(srcs[i], sls[i], anchors0)
+        torch.cuda.synchronize()
+        res = {}
+        for name, fn in (("pack", lambda i: traj.gc.pack_anchors(srcs[i % 4], sls[i % 4], anchors0)),
+                         ("unpack", lambda i: traj.gc.unpack_anchors(sls[i % 4], srcs[i % 4], anchors0))):
+            gpk = torch.cuda.CUDAGraph()  # launched from a graph: the copies, not the host, are timed
+            with torch.cuda.graph(gpk):
+                for i in range(reps):
+                    fn(i)
+            gpk.replay()
+            p0, p1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            p0.record()
+            gpk.replay()
+            p1.record()
+            torch.cuda.synchronize()
+            us = p0.elapsed_time(p1) * 1e3 / reps
+            nbytes = 2 * sls[0].numel() * sls[0].element_size()
+            res[name] = {"us_per_call": us, "GBs": nbytes / us / 1e3,
+                         "frac_of_peak": nbytes / us / 1e3 / measured_peak()[0]}
+        pack = {"what": "anchor rows (%d of %d views) of the bf16 latents, %d assets" % (len(anchors0), w.N, w.B),
+                **res}
+        del srcs, sls
+
     e2e = None
     if not args.no_e2e:
         host = traj.host_inputs()
@@ -500,6 +536,7 @@ def main():
                      "avg_launch_us": 1e3 * k_avg_ms, "launches": len(kernel_ms),
                      "frac_of_8TBs": achieved / 8000.0},
         "gpu_launches": launches,
+        "pack_anchors": pack,
         "clocks": clocks.summary(),
         "e2e": e2e,
     }

@@ -239,6 +239,27 @@ int geocache_reconstruct(const void* x_t, const float* x0, void* x_next, geocach
                          int64_t n, const geocache_recon* recon, float* x0_store, void* stream);
 
 /* --------------------------------------------------------------------------
+ * geocache_pack_anchors / geocache_unpack_anchors -- the batch slicing around
+ * the denoiser's anchor-only forward (Sec. 3.2, batch-sliced anchor forward:
+ * at a cached step only the anchor rows of the batch run the denoiser, each
+ * keeping its own structural indices).
+ *
+ * A per-view tensor is seen as B x N rows of row_bytes bytes (e.g. latents
+ * [B,N,C,H,W], conditioning maps, or per-view index tensors).
+ *   pack:   dst [B, a, row] receives src [B, N, row] rows of the anchors, in
+ *           the order of `anchors` (host [a], ascending, distinct, in [0, N)).
+ *   unpack: dst [B, N, row] receives src [B, a, row] at the anchors' rows; the
+ *           other rows of dst are left untouched.
+ * Both are device copies of raw bytes (any dtype), asynchronous on `stream`;
+ * src and dst must not overlap.  Sizes: 0 <= B <= 65535, 1 <= a <= N <= 64,
+ * row_bytes >= 0.  Returns GEOCACHE_OK, EINVAL, ESHAPE, EALIAS, ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_pack_anchors(const void* src, void* dst, int64_t row_bytes, int B, int N, const int32_t* anchors, int a,
+                          void* stream);
+int geocache_unpack_anchors(const void* src, void* dst, int64_t row_bytes, int B, int N, const int32_t* anchors,
+                            int a, void* stream);
+
+/* --------------------------------------------------------------------------
  * geocache_is_full_step -- 1 if `step` (0 <= step < S) is a full step under
  * `sched`, 0 if cached, a negative status on bad arguments. Host only.
  * ------------------------------------------------------------------------ */

@@ -262,3 +262,19 @@ def denoiser_flops(S: int, N: int, a: int, sched: dict, per_step: float) -> floa
     """Denoiser cost of a schedule: a full step costs per_step, a cached step
     a/N of it (only the anchor rows run the denoiser)."""
     return sum(per_step if is_full_step(t, S, sched) else per_step * a / N for t in range(S))
+
+
+# ------------------------------------------------- anchor-row pack / unpack --
+def pack_anchors(src, anchors):
+    """Rows of the anchor views, in anchor order (Sec. 3.2, batch-sliced
+    anchor forward: the denoiser runs on the anchor rows only, each keeping
+    its structural indices).  src [B, N, ...] -> [B, a, ...]."""
+    src = np.asarray(src)
+    return src[:, list(anchors)].copy()
+
+
+def unpack_anchors(src, dst, anchors):
+    """Scatter of anchor rows back to their views: dst[:, anchors[s]] = src[:, s]."""
+    out = np.array(dst, copy=True)
+    out[:, list(anchors)] = np.asarray(src)
+    return out

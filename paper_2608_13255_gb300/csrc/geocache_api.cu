@@ -322,6 +322,40 @@ int geocache_reconstruct(const void* x_t, const float* x0, void* x_next, geocach
     return ok();
 }
 
+static int copy_rows_entry(const void* src, void* dst, int64_t row_bytes, int B, int N, const int32_t* anchors, int a,
+                           bool pack, void* stream) {
+    const char* fn = pack ? "geocache_pack_anchors" : "geocache_unpack_anchors";
+    if (B < 0 || B > 65535) return fail(GEOCACHE_ESHAPE, "%s: B=%d out of range [0, 65535]", fn, B);
+    if (N < 1 || N > GEOCACHE_MAX_VIEWS) return fail(GEOCACHE_ESHAPE, "%s: N=%d out of range [1, %d]", fn, N, GEOCACHE_MAX_VIEWS);
+    if (row_bytes < 0) return fail(GEOCACHE_ESHAPE, "%s: row_bytes=%lld is negative", fn, (long long)row_bytes);
+    if (!anchors) return fail(GEOCACHE_EINVAL, "%s: anchors is NULL", fn);
+    if (a < 1 || a > N) return fail(GEOCACHE_EINVAL, "%s: a=%d must be in [1, N=%d]", fn, a, N);
+    geocache::RowAnchors anc{};
+    for (int s2 = 0; s2 < a; ++s2) {
+        if (anchors[s2] < 0 || anchors[s2] >= N) return fail(GEOCACHE_EINVAL, "%s: anchor %d out of range", fn, anchors[s2]);
+        if (s2 && anchors[s2] <= anchors[s2 - 1])
+            return fail(GEOCACHE_EINVAL, "%s: anchors must be ascending and distinct", fn);
+        anc.v[s2] = anchors[s2];
+    }
+    const size_t full = (size_t)B * N * (size_t)row_bytes, part = (size_t)B * a * (size_t)row_bytes;
+    if (full && (!src || !dst)) return fail(GEOCACHE_EINVAL, "%s: src and dst are required", fn);
+    if (overlap(src, pack ? full : part, dst, pack ? part : full))
+        return fail(GEOCACHE_EALIAS, "%s: src and dst overlap", fn);
+    cudaError_t e = geocache::launch_copy_rows(src, dst, row_bytes, B, N, a, anc, pack, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
+int geocache_pack_anchors(const void* src, void* dst, int64_t row_bytes, int B, int N, const int32_t* anchors, int a,
+                          void* stream) {
+    return copy_rows_entry(src, dst, row_bytes, B, N, anchors, a, true, stream);
+}
+
+int geocache_unpack_anchors(const void* src, void* dst, int64_t row_bytes, int B, int N, const int32_t* anchors,
+                            int a, void* stream) {
+    return copy_rows_entry(src, dst, row_bytes, B, N, anchors, a, false, stream);
+}
+
 int geocache_is_full_step(int step, int S, const geocache_schedule* sched) {
     if (!sched) return fail(GEOCACHE_EINVAL, "schedule is NULL");
     if (S < 1 || step < 0 || step >= S) return fail(GEOCACHE_ESHAPE, "step=%d outside [0, S=%d)", step, S);

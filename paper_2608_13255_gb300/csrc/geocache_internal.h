@@ -47,6 +47,12 @@ struct TransportArgs {
     int32_t slot_of[GEOCACHE_MAX_VIEWS];   // slot in `anchors`, -1 for non-anchors
 };
 
+struct RowAnchors {
+    int32_t v[GEOCACHE_MAX_VIEWS];
+};
+cudaError_t launch_copy_rows(const void* src, void* dst, long long row_bytes, int B, int N, int a,
+                             const RowAnchors& anc, bool pack, cudaStream_t s);
+
 cudaError_t launch_tau(const float* pos, const uint8_t* valid, int B, int N, int H, int W,
                        float tol_frac, float* tau, cudaStream_t s);
 cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s);

@@ -1334,6 +1334,51 @@ cudaError_t launch_copy_anchor_rows(const TransportArgs& t, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+// ------------------------------------------------- anchor-row pack / unpack --
+// Gather (pack) of the anchor views' rows of a per-view tensor [B, N, row]
+// into [B, a, row] in anchor order, and the scatter back (unpack): the batch
+// slicing around the denoiser's anchor-only forward (Sec. 3.2).  Rows are
+// copied as raw bytes, 16 bytes per thread when sizes and addresses allow.
+template <int VB>
+__global__ void __launch_bounds__(256) copy_rows_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
+                                                        long long row_bytes, int N, int a, RowAnchors anc, int pack) {
+    const int s = blockIdx.y, b = blockIdx.z;
+    const int u = anc.v[s];
+    const long long src_row = pack ? (long long)b * N + u : (long long)b * a + s;
+    const long long dst_row = pack ? (long long)b * a + s : (long long)b * N + u;
+    const uint8_t* sp = src + src_row * row_bytes;
+    uint8_t* dp = dst + dst_row * row_bytes;
+    const long long n = row_bytes / VB;
+    for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (long long)gridDim.x * blockDim.x) {
+        if (VB == 16)
+            __stcs(reinterpret_cast<uint4*>(dp) + i, __ldcs(reinterpret_cast<const uint4*>(sp) + i));
+        else if (VB == 4)
+            __stcs(reinterpret_cast<uint32_t*>(dp) + i, __ldcs(reinterpret_cast<const uint32_t*>(sp) + i));
+        else
+            dp[i] = sp[i];
+    }
+}
+
+cudaError_t launch_copy_rows(const void* src, void* dst, long long row_bytes, int B, int N, int a,
+                             const RowAnchors& anc, bool pack, cudaStream_t s) {
+    if (row_bytes == 0 || B == 0 || a == 0) return cudaSuccess;
+    const uintptr_t al = (uintptr_t)src | (uintptr_t)dst | (uintptr_t)row_bytes;
+    const int vb = al % 16 == 0 ? 16 : (al % 4 == 0 ? 4 : 1);
+    const long long n = row_bytes / vb;
+    long long gx = (n + 255) / 256;
+    if (gx > 1024) gx = 1024;
+    dim3 grid((unsigned)gx, a, B);
+    const uint8_t* sp = static_cast<const uint8_t*>(src);
+    uint8_t* dp = static_cast<uint8_t*>(dst);
+    if (vb == 16)
+        copy_rows_kernel<16><<<grid, 256, 0, s>>>(sp, dp, row_bytes, N, a, anc, pack);
+    else if (vb == 4)
+        copy_rows_kernel<4><<<grid, 256, 0, s>>>(sp, dp, row_bytes, N, a, anc, pack);
+    else
+        copy_rows_kernel<1><<<grid, 256, 0, s>>>(sp, dp, row_bytes, N, a, anc, pack);
+    return cudaGetLastError();
+}
+
 // ---------------------------------------------------- full-step recon --
 // Elementwise x_t, x0 -> x_next (and optionally pred, a copy of x0), four
 // consecutive elements per thread with 16-byte accesses when every pointer

@@ -67,8 +67,8 @@ assert ctypes.sizeof(Camera) == 64
 _LIB = None
 EXPORTS = ("geocache_build_corr", "geocache_transport_step", "geocache_reconstruct", "geocache_is_full_step",
            "geocache_rotate_anchors", "geocache_device_status", "geocache_corr_record_count",
-           "geocache_transport_workspace", "geocache_transport_step_noalloc", "geocache_last_error",
-           "geocache_abi_version")
+           "geocache_transport_workspace", "geocache_transport_step_noalloc", "geocache_pack_anchors",
+           "geocache_unpack_anchors", "geocache_last_error", "geocache_abi_version")
 
 
 def lib_path() -> str:
@@ -91,6 +91,9 @@ def load():
         L.geocache_transport_step_noalloc.argtypes = [ctypes.POINTER(Corr), P, i, i, P, P, P, P, P, i,
                                                       ctypes.POINTER(Recon), P]
         L.geocache_transport_step_noalloc.restype = ctypes.c_int
+        for name in ("geocache_pack_anchors", "geocache_unpack_anchors"):
+            getattr(L, name).argtypes = [P, P, i64, i, i, P, i, P]
+            getattr(L, name).restype = ctypes.c_int
         L.geocache_corr_record_count.argtypes = [ctypes.POINTER(Corr), ctypes.POINTER(ctypes.c_int64), P]
         L.geocache_corr_record_count.restype = ctypes.c_int
         L.geocache_transport_workspace.argtypes = [ctypes.POINTER(Corr), i]
@@ -317,6 +320,35 @@ def transport_step_noalloc(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev,
         _dev(x0_anchor_new, torch.float32, c.B * a * C * c.H * c.W, "x0_anchor_new"),
         _dev(x0_prev, torch.float32, n_all, "x0_prev"), _dev(x0_out, torch.float32, n_all, "x0_out"),
         pt, pn, lat, ctypes.byref(recon) if recon is not None else None, _stream(stream)))
+
+
+def _rows(src_full, a):
+    if src_full.dim() < 2:
+        raise ValueError("per-view tensors are [B, N, ...]")
+    B, N = src_full.shape[0], src_full.shape[1]
+    return B, N, (src_full[0, 0].numel() if B * N else 0) * src_full.element_size()
+
+
+def pack_anchors(src, dst, anchors, stream=None):
+    """geocache_pack_anchors: dst [B, a, ...] <- src[:, anchors] (raw bytes)."""
+    anc = sorted(int(x) for x in anchors)
+    B, N, row = _rows(src, len(anc))
+    if dst.dtype != src.dtype or tuple(dst.shape) != (B, len(anc)) + tuple(src.shape[2:]):
+        raise ValueError("dst must be [B, a, ...] of src's dtype")
+    arr = (ctypes.c_int32 * len(anc))(*anc)
+    _check(load().geocache_pack_anchors(_dev(src, src.dtype, name="src"), _dev(dst, dst.dtype, name="dst"), row, B, N,
+                                        ctypes.cast(arr, ctypes.c_void_p), len(anc), _stream(stream)))
+
+
+def unpack_anchors(src, dst, anchors, stream=None):
+    """geocache_unpack_anchors: dst[:, anchors] <- src [B, a, ...] (raw bytes)."""
+    anc = sorted(int(x) for x in anchors)
+    B, N, row = _rows(dst, len(anc))
+    if src.dtype != dst.dtype or tuple(src.shape) != (B, len(anc)) + tuple(dst.shape[2:]):
+        raise ValueError("src must be [B, a, ...] of dst's dtype")
+    arr = (ctypes.c_int32 * len(anc))(*anc)
+    _check(load().geocache_unpack_anchors(_dev(src, src.dtype, name="src"), _dev(dst, dst.dtype, name="dst"), row, B, N,
+                                          ctypes.cast(arr, ctypes.c_void_p), len(anc), _stream(stream)))
 
 
 def reconstruct(x_t, x0, x_next, recon: Recon, x0_store=None, stream=None):

@@ -252,3 +252,23 @@ def test_cost_model_reproduces_table1(row):
         sched = {"kind": "list", "steps": list(range(full - 1)) + [S - 1]}
     assert sum(oracle.is_full_step(t, S, sched) for t in range(S)) == full
     assert oracle.denoiser_flops(S, N, a, sched, per) == pytest.approx(printed, abs=0.006)
+
+
+# --------------------------------------------------- anchor-row pack / unpack --
+def test_pack_unpack_pins():
+    rng = np.random.default_rng(9)
+    x = rng.standard_normal((3, 6, 4, 5, 7))
+    A = [1, 4]
+    p = oracle.pack_anchors(x, A)
+    assert p.shape == (3, 2, 4, 5, 7)
+    for b in range(3):  # row by row, the definition
+        for s, u in enumerate(A):
+            np.testing.assert_array_equal(p[b, s], x[b, u])
+    # all views as anchors: identity; unpack inverts pack on the anchor rows and
+    # leaves the others untouched
+    np.testing.assert_array_equal(oracle.pack_anchors(x, range(6)), x)
+    y = rng.standard_normal(x.shape)
+    z = oracle.unpack_anchors(p, y, A)
+    np.testing.assert_array_equal(z[:, A], x[:, A])
+    others = [v for v in range(6) if v not in A]
+    np.testing.assert_array_equal(z[:, others], y[:, others])
