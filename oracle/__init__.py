@@ -61,7 +61,7 @@ def _lib():
         lib.oracle_reconstruct.argtypes = [_P, _P, _P, _P, l, i, d, d, d, d, i]
         lib.oracle_reconstruct.restype = i
         lib.oracle_transport_step.argtypes = [i, i, i, i, i, i, _P, _P, _P, _P, _P, _P, _P, i,
-                                              _P, _P, _P, _P, _P, _P, i, d, d, d, d, i, _P]
+                                              _P, _P, _P, _P, _P, _P, i, d, d, d, d, i, _P, i]
         lib.oracle_transport_step.restype = i
         lib.oracle_round_bf16.argtypes = [_P, _P, l]
         lib.oracle_round_bf16.restype = None
@@ -149,13 +149,17 @@ def reconstruct(x_t, x0, sampler, a_t=0.0, a_prev=0.0, sigma=0.0, sigma_next=0.0
 
 # ------------------------------------------------------------- transport --
 def transport_step(anchors, x0_new, x0_prev, *, K=4, table=None, geom=None,
-                   x_t=None, recon=None, sel=None):
+                   x_t=None, recon=None, sel=None, update="delta"):
     """One cached step (Eq. 1 + aggregation + loop order of Sec. 3.2).
 
     table = (idx, w) tables, or geom = (pos, valid, cams, tau).
     recon = dict(sampler=..., a_t=, a_prev=, sigma=, sigma_next=, pred_kind=) or None.
+    update = "delta" (Eq. 1) or "copy" (the value-copy ablation of Sec. 4.3:
+    covered targets take the anchors' transported x0).
     Returns (x0_out, x_next, pred) in binary64 (x_next/pred None without recon).
     """
+    if update not in ("delta", "copy"):
+        raise ValueError("update must be 'delta' or 'copy'")
     x0_new, x0_prev = _c(x0_new, np.float64), _c(x0_prev, np.float64)
     B, N, C, H, W = x0_prev.shape
     a = len(anchors)
@@ -182,10 +186,31 @@ def transport_step(anchors, x0_new, x0_prev, *, K=4, table=None, geom=None,
         B, N, H, W, K, C, _ptr(idx), _ptr(w), _ptr(pos), _ptr(valid), _ptr(cams), _ptr(tau_b),
         anc.ctypes.data, a, x0_new.ctypes.data, x0_prev.ctypes.data, x0_out.ctypes.data,
         _ptr(x_t if recon is not None else None), _ptr(x_next), _ptr(pred),
-        r["sampler"], r["a_t"], r["a_prev"], r["sigma"], r["sigma_next"], r["pred_kind"], _ptr(sel))
+        r["sampler"], r["a_t"], r["a_prev"], r["sigma"], r["sigma_next"], r["pred_kind"], _ptr(sel),
+        1 if update == "copy" else 0)
     if rc != 0:
         raise ValueError("oracle_transport_step: invalid arguments (%d)" % rc)
     return x0_out, x_next, pred
+
+
+def shuffle_rows(idx, w, perm):
+    """The shuffled-correspondence ablation of Sec. 4.3 ("corr -> shuffled")
+    on dense tables: the nonzero rows of every G_{u->v} (target tokens of view
+    v with a kept tap in view u), enumerated in (b, v, u, token) order, are
+    permuted: row number r takes the taps and weights of row number perm[r].
+    perm must map the rows of each (b, v, u) onto themselves.  Returns new
+    (idx, w); zero rows stay zero."""
+    idx, w = np.asarray(idx), np.asarray(w)
+    K = idx.shape[-1]
+    flat_i, flat_w = idx.reshape(-1, K), w.reshape(-1, K)
+    rows = np.flatnonzero((flat_i >= 0).any(axis=1))  # (b, v, u, token) order
+    perm = np.asarray(perm, dtype=np.int64)
+    if perm.shape != rows.shape:
+        raise ValueError("perm has %d entries for %d nonzero rows" % (perm.size, rows.size))
+    out_i, out_w = flat_i.copy(), flat_w.copy()
+    out_i[rows] = flat_i[rows[perm]]
+    out_w[rows] = flat_w[rows[perm]]
+    return out_i.reshape(idx.shape), out_w.reshape(w.shape)
 
 
 def round_bf16(x) -> np.ndarray:

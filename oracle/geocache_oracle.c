@@ -283,7 +283,11 @@ int oracle_reconstruct(const double* x_t, const double* x0, double* x_next, doub
  * computed from the geometry (pos/valid/cams/tau) with oracle_taps.
  * Layouts: x0_new [B,a,C,H,W]; x0_prev, x0_out, x_t, x_next, pred [B,N,C,H,W].
  * Only target pixels with sel[b*N*HW + v*HW + p] != 0 are written when sel
- * is given (sampled checks at large sizes). */
+ * is given (sampled checks at large sizes).
+ * copy != 0 is the value-copy ablation of Sec. 4.3 ("delta -> copy"): a
+ * covered target takes the anchors' transported x0 itself,
+ *     x0^v(t) = (1/n) sum_{u in A covering p} sum_k w_k(p) x0_new^u[q_k],
+ * and an uncovered one keeps x0^v(t-1). */
 int oracle_transport_step(int B, int N, int H, int W, int K, int C,
                           const int32_t* idx, const double* wtab,
                           const float* pos, const uint8_t* valid, const float* cams, const float* tau,
@@ -291,7 +295,7 @@ int oracle_transport_step(int B, int N, int H, int W, int K, int C,
                           const double* x0_new, const double* x0_prev, double* x0_out,
                           const double* x_t, double* x_next, double* pred,
                           int sampler, double a_t, double a_prev, double sigma, double sigma_next,
-                          int pred_kind, const uint8_t* sel) {
+                          int pred_kind, const uint8_t* sel, int copy) {
     if (a < 1 || a > N || C < 1 || (K != 1 && K != 4)) return -1;
     if (!idx && (!pos || !valid || !cams || !tau)) return -1;
     int slot_of[256];
@@ -345,14 +349,17 @@ int oracle_transport_step(int B, int N, int H, int W, int K, int C,
                             for (int k = 0; k < K; ++k) {
                                 if (ti[k] < 0) continue;
                                 const size_t q = (size_t)c * HW + (size_t)ti[k];
-                                g += tw[k] * (x0_new[nw + q] - x0_prev[pu + q]);
+                                /* Eq. 1 carries the anchor's change; the value-copy
+                                   ablation (Sec. 4.3) carries its x0 itself */
+                                g += tw[k] * (copy ? x0_new[nw + q] : x0_new[nw + q] - x0_prev[pu + q]);
                             }
                             acc[c] += g;
                         }
                     }
                     for (int c = 0; c < C; ++c)
-                        x0_out[plane0 + c * HW] = n ? x0_prev[plane0 + c * HW] + acc[c] / n
-                                                    : x0_prev[plane0 + c * HW];
+                        x0_out[plane0 + c * HW] = !n    ? x0_prev[plane0 + c * HW]
+                                                  : copy ? acc[c] / n
+                                                         : x0_prev[plane0 + c * HW] + acc[c] / n;
                 }
                 if (x_t && x_next)
                     for (int c = 0; c < C; ++c) {

@@ -436,6 +436,20 @@ def delta(w: Workload, step: int, views, std: float = 0.1) -> np.ndarray:
     return out
 
 
+def pair_permutation(pair_counts, seed: int) -> np.ndarray:
+    """Seeded input of the shuffled-correspondence ablation: a permutation of
+    the records (int32) that maps the records of each (b, v, u) pair onto
+    themselves; pair_counts[i] = records of pair i in (b, v, u) order."""
+    counts = np.asarray(pair_counts, np.int64).reshape(-1)
+    perm = np.empty(int(counts.sum()), np.int32)
+    rng = _rng(0x5AFF1E, seed)
+    start = 0
+    for n in counts:
+        perm[start:start + n] = start + rng.permutation(int(n))
+        start += int(n)
+    return perm
+
+
 def to_bf16_bits(x: np.ndarray) -> np.ndarray:
     """Round float32 to bfloat16 (round-to-nearest-even, via torch) and return
     the raw 16-bit patterns as uint16."""
