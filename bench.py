@@ -98,6 +98,52 @@ def step_bytes(w):
     return non + anc
 
 
+def measure_ablations(traj, reps=24):
+    """Cached-step time of the two ablation modes of Sec. 4.3 (value copy,
+    shuffled correspondence) beside the delta transport, on the bench's
+    workload and first cached anchor set: each graph runs `reps` steps
+    ping-ponging the x0 cache (every step reads and writes more than the L2
+    holds).  Sparse mode only."""
+    import torch
+    from paper_2608_13255_gb300 import synth
+    gc, w = traj.gc, traj.w
+    t0 = next(iter(traj.anchor_x0))
+    anchors = sorted(gc.rotate_anchors(w.N, w.a, t0, w.S, traj.sched)[0])
+    T = gc.tiles_per_view(w.H, w.W)
+    tp = traj.corr._keep["tile_ptr"].cpu().numpy().astype(np.int64)
+    perm = torch.from_numpy(synth.pair_permutation(tp[T::T] - tp[:-1:T], seed=1)).to(traj.dev)
+    shuffled = gc.permute_records(traj.corr, perm)
+    hw, lb = w.H * w.W, (2 if w.dtype == "bf16" else 4)
+    variants = (("delta", traj.corr, "delta", step_bytes(w)),
+                ("value_copy", traj.corr, "copy", step_bytes(w) - w.B * w.a * w.C * hw * 4),
+                ("shuffled", shuffled, "delta", step_bytes(w)))
+    out = {}
+    for name, corr, update, nbytes in variants:
+        def one(i):
+            src, dst = traj.bufs[i % 2], traj.bufs[(i + 1) % 2]
+            gc.transport_step(corr, anchors, w.C, traj.anchor_x0[t0], src, dst, traj.x, traj.x, traj.recon[t0],
+                              workspace=traj.workspace, update=update)
+        for i in range(2):
+            one(i)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for i in range(reps):
+                one(i)
+        g.replay()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) * 1e3 / reps
+        out[name] = {"us_per_step": us, "alg_bytes": nbytes, "GBs": nbytes / us / 1e3,
+                     "frac_of_peak": nbytes / us / 1e3 / measured_peak()[0]}
+    gc.device_status()
+    out["what"] = ("one cached step, %d assets, anchors %s, %d steps per graph; value_copy reads no anchor "
+                   "x0(t-1); shuffled = records permuted within each (b, v, u) pair (seed 1)" % (w.B, anchors, reps))
+    return out
+
+
 class Trajectory:
     """Device state of one batch's trajectory and the loop over its steps."""
 
@@ -504,6 +550,8 @@ def main():
                 **res}
         del srcs, sls
 
+    ablations = measure_ablations(traj) if rank == 0 and args.corr == "sparse" else None
+
     e2e = None
     if not args.no_e2e:
         host = traj.host_inputs()
@@ -537,6 +585,7 @@ def main():
                      "frac_of_8TBs": achieved / 8000.0},
         "gpu_launches": launches,
         "pack_anchors": pack,
+        "ablations": ablations,
         "clocks": clocks.summary(),
         "e2e": e2e,
     }

@@ -69,6 +69,13 @@ typedef enum {
                                    them record-parallel into a workspace (fastest) */
 } geocache_corr_mode;
 
+/* Update rule of the views outside the anchor set at a cached step. */
+typedef enum {
+    GEOCACHE_UPDATE_DELTA = 0, /* Eq. 1: integrate the anchors' transported change of x0 */
+    GEOCACHE_UPDATE_COPY = 1   /* value-copy ablation (Sec. 4.3, Table 3 "delta -> copy"): a covered
+                                  token takes the anchors' transported x0 itself */
+} geocache_update;
+
 /* One kept (target token, source view) row of G_{u->v} in sparse form: the
  * bilinear footprint's top-left tap and fractions, from which the kept taps'
  * indices and renormalised weights follow exactly as in the tables.
@@ -227,6 +234,45 @@ int geocache_transport_step(const geocache_corr* corr, const int32_t* anchors, i
                             void* stream);
 
 /* --------------------------------------------------------------------------
+ * geocache_transport_step_update -- geocache_transport_step with the update
+ * rule of the views outside the anchor set chosen (the ablations of Sec. 4.3).
+ * GEOCACHE_UPDATE_DELTA is geocache_transport_step.  GEOCACHE_UPDATE_COPY
+ * overwrites instead of integrating: a token of view v with n >= 1 covering
+ * anchors gets
+ *     x0_out^v = (1/n) sum_{u in A with a kept tap} sum_k w_k x0_anchor_new^u[q_k]
+ * and a token with n = 0 keeps x0_prev^v; anchors and the reconstruction are
+ * as in geocache_transport_step.  Same arguments, layouts, ownership and
+ * statuses as geocache_transport_step, plus EINVAL for an unknown update.
+ * ------------------------------------------------------------------------ */
+int geocache_transport_step_update(const geocache_corr* corr, geocache_update update, const int32_t* anchors, int a,
+                                   int C, const float* x0_anchor_new, const float* x0_prev, float* x0_out,
+                                   const void* x_t, void* x_next, geocache_dtype lat_dtype,
+                                   const geocache_recon* recon, float* workspace, int64_t workspace_floats,
+                                   void* stream);
+
+/* --------------------------------------------------------------------------
+ * geocache_permute_records -- the shuffled-correspondence ablation (Sec. 4.3,
+ * Table 3 "corr -> shuffled"): the nonzero rows of each G_{u->v} exchange
+ * their taps.  out[r] keeps the target token of corr->records[r] and takes
+ * the keep mask, top-left tap and fractions of corr->records[perm[r]], for
+ * r in [0, corr->max_records).
+ *   corr   a sparse-form corr filled by geocache_build_corr (records,
+ *          max_records; its other fields are not read).
+ *   perm   device [max_records] i32, a permutation of [0, max_records) that
+ *          maps the records of each (b, v, u) pair, tile_ptr[i*T] ..
+ *          tile_ptr[(i+1)*T) with i = (b*N + v)*N + u, onto themselves (the
+ *          caller's seeded input; other permutations give a correspondence
+ *          whose rows belong to other pairs).  An entry outside
+ *          [0, max_records) leaves out[r] = records[r] and sets the device
+ *          status word (geocache_device_status then returns EINVAL).
+ *   out    device [max_records] records, 16-byte aligned, overlapping
+ *          neither corr->records nor perm.  A corr whose records are `out`
+ *          runs the shuffled transport in GEOCACHE_CORR_SPARSE mode.
+ * Asynchronous.  Returns GEOCACHE_OK, EINVAL, EALIAS, ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_permute_records(const geocache_corr* corr, const int32_t* perm, geocache_tap_record* out, void* stream);
+
+/* --------------------------------------------------------------------------
  * geocache_reconstruct -- full-step passthrough (Sec. 3.2: at a full step the
  * denoiser runs on all N views and its x0 is both the new reference and the
  * input of the sampler conversion).
@@ -287,9 +333,11 @@ int geocache_rotate_anchors(int N, int a, int step, int S, const geocache_schedu
  * device status word.  Failures only the GPU can see set it instead of
  * trapping, so the context stays usable: a sparse-form build whose records
  * exceed max_records (the excess is dropped; transport steps read only the
- * records that exist), and a bounded wait inside a kernel that ran out (its
- * CTA returns without writing its outputs).  Returns GEOCACHE_OK, ESHAPE
- * (record overflow), ETIMEOUT (a wait gave up) or ECUDA.
+ * records that exist), a record permutation entry out of range
+ * (geocache_permute_records keeps that record), and a bounded wait inside a
+ * kernel that ran out (its CTA returns without writing its outputs).
+ * Returns GEOCACHE_OK, ESHAPE (record overflow), EINVAL (bad permutation
+ * entry), ETIMEOUT (a wait gave up) or ECUDA.
  * ------------------------------------------------------------------------ */
 int geocache_device_status(void* stream);
 

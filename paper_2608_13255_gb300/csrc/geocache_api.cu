@@ -122,6 +122,9 @@ int geocache_device_status(void* stream) {
     if (word & 2u)
         return fail(GEOCACHE_ESHAPE, "a sparse-form build had more records than max_records (status word 0x%x); "
                                      "query geocache_corr_record_count and rebuild", word);
+    if (word & 4u)
+        return fail(GEOCACHE_EINVAL, "a record permutation entry was outside [0, max_records) (status word 0x%x); "
+                                     "those records were kept", word);
     if (word) return fail(GEOCACHE_ETIMEOUT, "a bounded device wait gave up (status word 0x%x); outputs of that call are incomplete", word);
     return ok();
 }
@@ -205,7 +208,18 @@ int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int 
                             const float* x0_anchor_new, const float* x0_prev, float* x0_out, const void* x_t,
                             void* x_next, geocache_dtype lat_dtype, const geocache_recon* recon, float* workspace,
                             int64_t workspace_floats, void* stream) {
+    return geocache_transport_step_update(c, GEOCACHE_UPDATE_DELTA, anchors, a, C, x0_anchor_new, x0_prev, x0_out,
+                                          x_t, x_next, lat_dtype, recon, workspace, workspace_floats, stream);
+}
+
+int geocache_transport_step_update(const geocache_corr* c, geocache_update update, const int32_t* anchors, int a,
+                                   int C, const float* x0_anchor_new, const float* x0_prev, float* x0_out,
+                                   const void* x_t, void* x_next, geocache_dtype lat_dtype,
+                                   const geocache_recon* recon, float* workspace, int64_t workspace_floats,
+                                   void* stream) {
     if (!c) return fail(GEOCACHE_EINVAL, "corr is NULL");
+    if (update != GEOCACHE_UPDATE_DELTA && update != GEOCACHE_UPDATE_COPY)
+        return fail(GEOCACHE_EINVAL, "unknown update rule %d", (int)update);
     int st = check_sizes(c->B, c->N, c->H, c->W);
     if (st) return st;
     if (c->K != 1 && c->K != 4) return fail(GEOCACHE_EINVAL, "K=%d must be 1 or 4", c->K);
@@ -272,6 +286,7 @@ int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int 
     // written, so an in-place update needs no separate anchor-row pass
     t.write_anchor_rows = (x0_out != x0_prev) || c->mode == GEOCACHE_CORR_SPARSE;
     t.lat_dtype = lat_dtype;
+    t.update = update;
     t.pos = c->pos; t.valid = c->valid; t.cams = c->cams; t.tau = c->tau; t.idx = c->idx; t.w = c->w;
     t.keep = c->keep;
     t.tile_ptr = c->tile_ptr;
@@ -292,6 +307,18 @@ int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int 
         e = geocache::launch_copy_anchor_rows(t, s);
         if (e != cudaSuccess) return cuda_fail(e, "anchor-row copy launch");
     }
+    return ok();
+}
+
+int geocache_permute_records(const geocache_corr* c, const int32_t* perm, geocache_tap_record* out, void* stream) {
+    if (!c || !perm || !out) return fail(GEOCACHE_EINVAL, "corr, perm and out are required");
+    if (!c->records || c->max_records < 0) return fail(GEOCACHE_EINVAL, "corr has no sparse records");
+    if (((uintptr_t)out | (uintptr_t)c->records) & 15) return fail(GEOCACHE_EINVAL, "records must be 16-byte aligned");
+    const size_t rb = (size_t)c->max_records * 16, pb = (size_t)c->max_records * 4;
+    if (overlap(out, rb, c->records, rb) || overlap(out, rb, perm, pb))
+        return fail(GEOCACHE_EALIAS, "out overlaps the records or the permutation");
+    cudaError_t e = geocache::launch_permute_records(c->records, perm, out, c->max_records, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "record permutation kernel launch");
     return ok();
 }
 

@@ -25,6 +25,7 @@ struct TransportArgs {
     int mode;                           // geocache_corr_mode
     int write_anchor_rows;              // 0 when x0_out aliases x0_prev (rows written afterwards)
     int lat_dtype;                      // geocache_dtype
+    int update;                         // geocache_update (Eq. 1 or the value-copy ablation)
     const float* pos;
     const uint8_t* valid;
     const geocache_camera* cams;
@@ -60,6 +61,8 @@ cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s);
 // tile_ptr (tile_ptr[n] = total, or -1 when the total exceeds INT32_MAX)
 cudaError_t launch_tile_ptr(const geocache_corr& c, cudaStream_t s);
 cudaError_t launch_fill_records(const geocache_corr& c, cudaStream_t s);
+cudaError_t launch_permute_records(const geocache_tap_record* src, const int32_t* perm, geocache_tap_record* dst,
+                                   long long n, cudaStream_t s);
 __host__ __device__ int tiles_per_view(int H, int W);
 cudaError_t launch_transport(const TransportArgs& t, cudaStream_t s);
 int transport_launch_count(int a, int C, int in_place);

@@ -41,6 +41,21 @@ __device__ __forceinline__ float recon_one(const ReconCoef& c, float xt, float x
     }
 }
 
+// One kept tap's term of an anchor's transported quantity, accumulated in
+// tap order: Eq. 1 carries the anchor's change x0_new - x0(t-1); the
+// value-copy ablation (Sec. 4.3, "delta -> copy") carries x0_new itself.
+__device__ __forceinline__ float tap_term(bool copy, float w, float xn, float xp, float acc) {
+    return __fmaf_rn(w, copy ? xn : __fsub_rn(xn, xp), acc);
+}
+
+// x0(t) of a covered target from x0(t-1) and the anchor-ordered sum g of its
+// n covering anchors' terms: x0 + g/n (Eq. 1, normalised multi-anchor sum),
+// or g/n under the value copy.
+__device__ __forceinline__ float fold_one(bool copy, float x0, float g, int n) {
+    const float m = n == 1 ? g : __fdiv_rn(g, (float)n);
+    return copy ? m : __fadd_rn(x0, m);
+}
+
 // -------------------------------------------------------------------- tau --
 // One thread-block cluster per asset: CTA r of the cluster reduces the
 // componentwise min / max of the foreground texels of views r, r + CS, ...
@@ -224,7 +239,8 @@ cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s) {
 }
 
 // Device status word (the library's only device-resident state): bit 0 = a
-// bounded wait gave up, bit 1 = the sparse form did not fit max_records.
+// bounded wait gave up, bit 1 = the sparse form did not fit max_records,
+// bit 2 = a record permutation entry was out of range.
 // Read and cleared by geocache_device_status().
 __device__ unsigned int g_device_error = 0;
 
@@ -616,6 +632,7 @@ __device__ __forceinline__ void item_increment(const TransportArgs& args, const 
     const int N = args.N, C = args.C, a = args.a;
     const float* xn = args.x0_new + (((size_t)b * a + s2) * C + cg) * plane;
     const float* xp = args.x0_prev + (((size_t)b * N + args.anchors[s2]) * C + cg) * plane;
+    const bool copy = args.update == GEOCACHE_UPDATE_COPY;
     float dn[K][4], dp[K][4];
 #pragma unroll
     for (int kk = 0; kk < K; ++kk)
@@ -634,7 +651,7 @@ __device__ __forceinline__ void item_increment(const TransportArgs& args, const 
         float acc = 0.0f;
 #pragma unroll
         for (int kk = 0; kk < K; ++kk)
-            if (tp.q[kk] >= 0) acc = __fmaf_rn(tp.w[kk], __fsub_rn(dn[kk][c], dp[kk][c]), acc);
+            if (tp.q[kk] >= 0) acc = tap_term(copy, tp.w[kk], dn[kk][c], dp[kk][c], acc);
         g[c] = acc;
     }
 }
@@ -840,7 +857,7 @@ __global__ void __launch_bounds__(kThreads) transport_fused_kernel(const Transpo
                     const float gg[4] = {g.x, g.y, g.z, g.w};
 #pragma unroll
                     for (int cc = 0; cc < 4; ++cc)
-                        x0[cc][i] = __fadd_rn(x0[cc][i], n == 1 ? gg[cc] : __fdiv_rn(gg[cc], (float)n));
+                        x0[cc][i] = fold_one(args.update == GEOCACHE_UPDATE_COPY, x0[cc][i], gg[cc], n);
                 }
             }
             if (slot < 0 || args.write_anchor_rows) {
@@ -915,7 +932,7 @@ __global__ void __launch_bounds__(kThreads) transport_simple_kernel(const Transp
             const float gg[4] = {g.x, g.y, g.z, g.w};
 #pragma unroll
             for (int cc = 0; cc < 4; ++cc)
-                x0[cc][i] = __fadd_rn(x0[cc][i], n == 1 ? gg[cc] : __fdiv_rn(gg[cc], (float)n));
+                x0[cc][i] = fold_one(args.update == GEOCACHE_UPDATE_COPY, x0[cc][i], gg[cc], n);
         }
     }
     if (slot < 0 || args.write_anchor_rows) {
@@ -981,7 +998,7 @@ struct QuadRows {
     }
 
     // add the folded increments of the tile (mean over covering anchors)
-    __device__ __forceinline__ void fold(const float (*s_acc)[4], const uint8_t* s_n, int lp0) {
+    __device__ __forceinline__ void fold(const float (*s_acc)[4], const uint8_t* s_n, int lp0, bool copy) {
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const int n = s_n[lp0 + i];
@@ -989,7 +1006,7 @@ struct QuadRows {
             const float4 gq = *reinterpret_cast<const float4*>(s_acc[lp0 + i]);
             const float gg[4] = {gq.x, gq.y, gq.z, gq.w};
 #pragma unroll
-            for (int c = 0; c < 4; ++c) x0[c][i] = __fadd_rn(x0[c][i], n == 1 ? gg[c] : __fdiv_rn(gg[c], (float)n));
+            for (int c = 0; c < 4; ++c) x0[c][i] = fold_one(copy, x0[c][i], gg[c], n);
         }
     }
 
@@ -1029,7 +1046,8 @@ __device__ __forceinline__ int nonanchor_view(const TransportArgs& args, int vi)
 }
 
 // Records of one pair applied by one CTA slice (grid-stride over the pair's records).
-template <int K>
+// COPY: the value-copy ablation (no x0(t-1) gathers).
+template <int K, bool COPY>
 __device__ __forceinline__ void apply_records(const TransportArgs& args, int pair_id, int slice, int n_slices) {
     const int N = args.N, C = args.C, a = args.a;
     const int HW = args.H * args.W;
@@ -1064,7 +1082,7 @@ __device__ __forceinline__ void apply_records(const TransportArgs& args, int pai
                     if (tp.q[kk] >= 0 && c < cn) {
                         const size_t e = (size_t)(cg + c) * plane + tp.q[kk];
                         dn[kk][c] = __ldg(xn + e);
-                        dp[kk][c] = __ldg(xp + e);
+                        if (!COPY) dp[kk][c] = __ldg(xp + e);
                     }
                 }
             float g[4];
@@ -1073,7 +1091,7 @@ __device__ __forceinline__ void apply_records(const TransportArgs& args, int pai
                 float acc = 0.0f;
 #pragma unroll
                 for (int kk = 0; kk < K; ++kk)
-                    if (tp.q[kk] >= 0) acc = __fmaf_rn(tp.w[kk], __fsub_rn(dn[kk][c], dp[kk][c]), acc);
+                    if (tp.q[kk] >= 0) acc = tap_term(COPY, tp.w[kk], dn[kk][c], dp[kk][c], acc);
                 g[c] = acc;
             }
             if (cn == 4 && C % 4 == 0) {
@@ -1089,7 +1107,7 @@ __device__ __forceinline__ void apply_records(const TransportArgs& args, int pai
 
 // Phase A: n_apply record-slice CTAs and n_stream anchor-view CTAs (tiles of
 // kTileTokens tokens), interleaved evenly in block order.
-template <typename T, int K, bool VEC>
+template <typename T, int K, bool VEC, bool COPY>
 __global__ void __launch_bounds__(kThreads) sparse_phase_a_kernel(const TransportArgs args, int n_apply,
                                                                   int n_stream, int n_slices) {
     pdl_launch_dependents();
@@ -1099,7 +1117,7 @@ __global__ void __launch_bounds__(kThreads) sparse_phase_a_kernel(const Transpor
     const bool is_stream = (int)((k + 1) * n_stream / total) > s_before;
     if (!is_stream) {
         const int ai = (int)k - s_before;
-        apply_records<K>(args, ai / n_slices, ai % n_slices, n_slices);
+        apply_records<K, COPY>(args, ai / n_slices, ai % n_slices, n_slices);
         return;
     }
     const int n_tiles = tiles_per_view_dev(args.H, args.W);
@@ -1208,7 +1226,7 @@ __global__ void __launch_bounds__(kThreads) sparse_phase_b_kernel(const Transpor
             }
         }
         if (cnt > 0) {
-            q.fold(s_acc, s_n, 4 * t);
+            q.fold(s_acc, s_n, 4 * t, args.update == GEOCACHE_UPDATE_COPY);
             q.store(args, b, v, p0, cnt, cg, cn);
         }
         if (cg + 4 < C) __syncthreads();  // sums are rewritten by the next channel group
@@ -1229,10 +1247,15 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
     if (n_apply + n_stream > 0) {
         if (n_apply + n_stream > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
         const unsigned g = (unsigned)(n_apply + n_stream);
-        if (vec)
-            sparse_phase_a_kernel<T, K, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
+        const bool copy = t.update == GEOCACHE_UPDATE_COPY;
+        if (vec && !copy)
+            sparse_phase_a_kernel<T, K, true, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
+        else if (vec)
+            sparse_phase_a_kernel<T, K, true, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
+        else if (!copy)
+            sparse_phase_a_kernel<T, K, false, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
         else
-            sparse_phase_a_kernel<T, K, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
+            sparse_phase_a_kernel<T, K, false, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
@@ -1357,6 +1380,36 @@ __global__ void __launch_bounds__(256) copy_rows_kernel(const uint8_t* __restric
         else
             dp[i] = sp[i];
     }
+}
+
+// ---------------------------------------------------- shuffled records --
+// The shuffled-correspondence ablation (Sec. 4.3, "corr -> shuffled"): record
+// r keeps its target token and takes the taps (keep mask, top-left tap,
+// fractions) of record perm[r].  An entry outside [0, n) sets bit 2 of the
+// status word and leaves the record as it was.
+__global__ void __launch_bounds__(256) permute_records_kernel(const int4* __restrict__ src,
+                                                              const int32_t* __restrict__ perm, int4* __restrict__ dst,
+                                                              long long n) {
+    for (long long r = blockIdx.x * (long long)blockDim.x + threadIdx.x; r < n; r += (long long)gridDim.x * blockDim.x) {
+        const int4 own = __ldg(src + r);
+        const int p = __ldg(perm + r);
+        if (p < 0 || p >= n) {
+            atomicOr(&g_device_error, 4u);
+            dst[r] = own;
+            continue;
+        }
+        const int4 o = __ldg(src + p);
+        dst[r] = make_int4((int)(((uint32_t)own.x & 0x0fffffffu) | ((uint32_t)o.x & 0xf0000000u)), o.y, o.z, o.w);
+    }
+}
+
+cudaError_t launch_permute_records(const geocache_tap_record* src, const int32_t* perm, geocache_tap_record* dst,
+                                   long long n, cudaStream_t s) {
+    if (n <= 0) return cudaSuccess;
+    const long long blocks = (n + 255) / 256;
+    permute_records_kernel<<<(unsigned)(blocks < 65535 * 8 ? blocks : 65535 * 8), 256, 0, s>>>(
+        reinterpret_cast<const int4*>(src), perm, reinterpret_cast<int4*>(dst), n);
+    return cudaGetLastError();
 }
 
 cudaError_t launch_copy_rows(const void* src, void* dst, long long row_bytes, int B, int N, int a,

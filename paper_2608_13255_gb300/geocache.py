@@ -21,6 +21,7 @@ F32, BF16 = 0, 1
 DDIM, FM_EULER = 0, 1
 PRED_NONE, PRED_EPS, PRED_V, PRED_VELOCITY = 0, 1, 2, 3
 CORR_GEOMETRY, CORR_TABLE, CORR_MASK, CORR_SPARSE = 0, 1, 2, 3
+UPDATE_DELTA, UPDATE_COPY = 0, 1
 TILE_TOKENS = 1024
 SCHED_EVERY_K, SCHED_HEAD_MID_TAIL, SCHED_LIST, SCHED_ALL_FULL, SCHED_SINGLE_CACHED = 0, 1, 2, 3, 4
 MAX_VIEWS = 64
@@ -68,7 +69,8 @@ _LIB = None
 EXPORTS = ("geocache_build_corr", "geocache_transport_step", "geocache_reconstruct", "geocache_is_full_step",
            "geocache_rotate_anchors", "geocache_device_status", "geocache_corr_record_count",
            "geocache_transport_workspace", "geocache_transport_step_noalloc", "geocache_pack_anchors",
-           "geocache_unpack_anchors", "geocache_last_error", "geocache_abi_version")
+           "geocache_unpack_anchors", "geocache_transport_step_update", "geocache_permute_records",
+           "geocache_last_error", "geocache_abi_version")
 
 
 def lib_path() -> str:
@@ -91,6 +93,11 @@ def load():
         L.geocache_transport_step_noalloc.argtypes = [ctypes.POINTER(Corr), P, i, i, P, P, P, P, P, i,
                                                       ctypes.POINTER(Recon), P]
         L.geocache_transport_step_noalloc.restype = ctypes.c_int
+        L.geocache_transport_step_update.argtypes = [ctypes.POINTER(Corr), i, P, i, i, P, P, P, P, P, i,
+                                                     ctypes.POINTER(Recon), P, i64, P]
+        L.geocache_transport_step_update.restype = ctypes.c_int
+        L.geocache_permute_records.argtypes = [ctypes.POINTER(Corr), P, P, P]
+        L.geocache_permute_records.restype = ctypes.c_int
         for name in ("geocache_pack_anchors", "geocache_unpack_anchors"):
             getattr(L, name).argtypes = [P, P, i64, i, i, P, i, P]
             getattr(L, name).restype = ctypes.c_int
@@ -274,9 +281,14 @@ def build_corr(corr: CorrHandle, stream=None) -> CorrHandle:
     return corr
 
 
+UPDATES = {"delta": UPDATE_DELTA, "copy": UPDATE_COPY}
+
+
 def transport_step(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev, x0_out, x_t=None, x_next=None,
-                   recon: Recon | None = None, workspace=None, stream=None):
-    """geocache_transport_step on torch tensors (see include/geocache.h)."""
+                   recon: Recon | None = None, workspace=None, stream=None, update="delta"):
+    """geocache_transport_step (update="delta", Eq. 1) or
+    geocache_transport_step_update (update="copy", the value-copy ablation)
+    on torch tensors (see include/geocache.h)."""
     c = corr.c
     anc = sorted(int(a) for a in anchors)
     a = len(anc)
@@ -289,14 +301,33 @@ def transport_step(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev, x0_out,
         dt = x_t.dtype
         pt, pn = _dev(x_t, dt, n_all, "x_t"), _dev(x_next, dt, n_all, "x_next")
         _check_pred(recon, n_all)
-    st = load().geocache_transport_step(
-        ctypes.byref(c), ctypes.cast(arr, ctypes.c_void_p), a, int(C),
+    st = load().geocache_transport_step_update(
+        ctypes.byref(c), UPDATES[update], ctypes.cast(arr, ctypes.c_void_p), a, int(C),
         _dev(x0_anchor_new, torch.float32, c.B * a * C * c.H * c.W, "x0_anchor_new"),
         _dev(x0_prev, torch.float32, n_all, "x0_prev"), _dev(x0_out, torch.float32, n_all, "x0_out"),
         pt, pn, lat, ctypes.byref(recon) if recon is not None else None,
         _dev(workspace, torch.float32, None, "workspace"), 0 if workspace is None else workspace.numel(),
         _stream(stream))
     _check(st)
+
+
+def permute_records(corr: CorrHandle, perm, out=None, stream=None) -> CorrHandle:
+    """geocache_permute_records (shuffled-correspondence ablation): a new
+    sparse-mode handle over `out` (allocated like corr's records when None)
+    whose rows exchange their taps by `perm` (device int32 [max_records])."""
+    c = corr.c
+    recs = corr._keep["records"]
+    if out is None:
+        out = torch.empty_like(recs)
+    _check(load().geocache_permute_records(ctypes.byref(c), _dev(perm, torch.int32, c.max_records, "perm"),
+                                           _dev(out, torch.int32, 4 * c.max_records, "out"), _stream(stream)))
+    refs = dict(corr._keep)
+    refs["records"] = out
+    refs["perm"] = perm
+    c2 = Corr.from_buffer_copy(c)
+    c2.records = out.data_ptr()
+    c2.mode = CORR_SPARSE
+    return CorrHandle(c2, refs)
 
 
 def transport_step_noalloc(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev, x0_out, x_t=None, x_next=None,

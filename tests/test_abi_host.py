@@ -131,3 +131,19 @@ def test_argument_errors_before_launch(gc):
     s, _k = gc.make_schedule({"kind": "every_k", "k": 5})
     assert L.geocache_rotate_anchors(6, 7, 1, 10, ctypes.byref(s), ctypes.cast(out, ctypes.c_void_p), None) == gc.EINVAL
     assert gc.last_error() != ""
+
+
+def test_ablation_entry_points_check_arguments(gc):
+    L = gc.load()
+    c = gc.Corr(1, 6, 8, 8, 4, 0.01, 16, 16, 16, 16, None, None, None, None, None, 0, gc.CORR_SPARSE)
+    anc = (ctypes.c_int32 * 2)(0, 3)
+    st = L.geocache_transport_step_update(ctypes.byref(c), 7, ctypes.cast(anc, ctypes.c_void_p), 2, 4, 16, 16, 32,
+                                          None, None, 0, None, None, 0, None)
+    assert st == gc.EINVAL and "update" in gc.last_error()
+    # the permutation needs records, a permutation and an output
+    assert L.geocache_permute_records(None, 16, 32, None) == gc.EINVAL
+    assert L.geocache_permute_records(ctypes.byref(c), 16, 32, None) == gc.EINVAL
+    assert "records" in gc.last_error()
+    c.records, c.max_records = 4096, 64
+    assert L.geocache_permute_records(ctypes.byref(c), 16, 4096 + 512, None) == gc.EALIAS  # out overlaps records
+    assert L.geocache_permute_records(ctypes.byref(c), 16, 4100, None) == gc.EINVAL  # misaligned out
