@@ -63,6 +63,8 @@ def _lib():
         lib.oracle_transport_step.argtypes = [i, i, i, i, i, i, _P, _P, _P, _P, _P, _P, _P, i,
                                               _P, _P, _P, _P, _P, _P, i, d, d, d, d, i, _P, i]
         lib.oracle_transport_step.restype = i
+        lib.oracle_raster.argtypes = [_P, i, _P, i, _P, i, i, _P, _P]
+        lib.oracle_raster.restype = i
         lib.oracle_round_bf16.argtypes = [_P, _P, l]
         lib.oracle_round_bf16.restype = None
         _LIB = lib
@@ -211,6 +213,30 @@ def shuffle_rows(idx, w, perm):
     out_i[rows] = flat_i[rows[perm]]
     out_w[rows] = flat_w[rows[perm]]
     return out_i.reshape(idx.shape), out_w.reshape(w.shape)
+
+
+def raster(V, F, cam, H, W):
+    """Position map [H,W,3] f32 and validity [H,W] u8 of mesh (V [nv,3]
+    world, F [nf,3] vertex indices) seen by camera `cam` (16 floats): the
+    nearest face whose projection contains the pixel centre, ties to the
+    lower face index; decisions and position in binary32 (Sec. 3.1 position
+    maps; see oracle_raster)."""
+    V = _c(V, np.float32)
+    F = _c(F, np.int32)
+    cam = _c(cam, np.float32)
+    pos = np.zeros((H, W, 3), np.float32)
+    valid = np.zeros((H, W), np.uint8)
+    rc = _lib().oracle_raster(V.ctypes.data, V.shape[0], F.ctypes.data, F.shape[0], cam.ctypes.data, H, W,
+                              pos.ctypes.data, valid.ctypes.data)
+    if rc != 0:
+        raise ValueError("oracle_raster: %d" % rc)
+    return pos, valid
+
+
+def raster_views(V, F, cams, H, W):
+    """raster() for each camera of cams [N,16]: ([N,H,W,3], [N,H,W])."""
+    out = [raster(V, F, c, H, W) for c in np.asarray(cams).reshape(-1, 16)]
+    return np.stack([o[0] for o in out]), np.stack([o[1] for o in out])
 
 
 def round_bf16(x) -> np.ndarray:

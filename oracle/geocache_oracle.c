@@ -410,3 +410,134 @@ static uint16_t bf16_from_double(double x) {
 void oracle_round_bf16(const double* x, uint16_t* out, long n) {
     for (long i = 0; i < n; ++i) out[i] = bf16_from_double(x[i]);
 }
+
+/* ------------------------------------------------------ position maps -- */
+/* The rendered position map of one mesh seen by one camera (Sec. 3.1: the
+ * per-pixel 3-D coordinates a geometry-conditioned texturing pipeline renders
+ * for each view, from which the correspondence operator of Sec. 3.2 is
+ * built).  A plain face-major z-buffer:
+ *   - a face is skipped when a vertex is not in front (camera z <= 1e-6) or
+ *     its projected signed area is 0;
+ *   - pixel (i, j) is covered when its centre (i + 0.5, j + 0.5) lies inside
+ *     or on the projected triangle: the three edge functions, each zero on
+ *     one edge, all have the sign of the area;
+ *   - its depth is the camera z of the intersection of the ray through the
+ *     centre with the face's plane, which must be positive;
+ *   - the nearest face wins, ties going to the lower face index;
+ *   - the stored position is that intersection in world coordinates.
+ * Every step is binary32, one rounding per operation in the order written
+ * (the decisions are the rasteriser's own; the position is exact to those
+ * roundings).  V [nv,3] world, F [nf,3] vertex indices, cam 16 floats;
+ * pos_out [H,W,3], valid_out [H,W].  Faces with an index outside [0, nv)
+ * are skipped.  Returns 0, or -1 on bad arguments, -2 on allocation failure. */
+typedef struct {
+    float R[9], t[3], fx, fy, cx, cy;
+} orc_cam32;
+
+static void raster_cam_point(const orc_cam32* c, const float* X, float* xc) {
+    for (int r = 0; r < 3; ++r) {
+        float s = c->R[3 * r] * X[0];
+        s = s + c->R[3 * r + 1] * X[1];
+        s = s + c->R[3 * r + 2] * X[2];
+        xc[r] = s + c->t[r];
+    }
+}
+
+/* depth of the ray through (pu, pv) on the plane (n, nd); 0 when there is none */
+static float raster_depth(const orc_cam32* c, const float* n, float nd, float pu, float pv, float* d) {
+    d[0] = (pu - c->cx) / c->fx;
+    d[1] = (pv - c->cy) / c->fy;
+    d[2] = 1.0f;
+    float den = n[0] * d[0];
+    den = den + n[1] * d[1];
+    den = den + n[2];
+    if (den == 0.0f) return 0.0f;
+    const float s = nd / den;
+    return (s > 0.0f && s <= 3.0e38f) ? s : 0.0f;
+}
+
+int oracle_raster(const float* V, int nv, const int32_t* F, int nf, const float* cam, int H, int W,
+                  float* pos_out, uint8_t* valid_out) {
+    if (!V || !F || !cam || !pos_out || !valid_out || nv < 0 || nf < 0 || H <= 0 || W <= 0) return -1;
+    orc_cam32 c;
+    for (int i = 0; i < 9; ++i) c.R[i] = cam[i];
+    for (int i = 0; i < 3; ++i) c.t[i] = cam[9 + i];
+    c.fx = cam[12]; c.fy = cam[13]; c.cx = cam[14]; c.cy = cam[15];
+    const size_t HW = (size_t)H * W;
+    float* depth = (float*)malloc(sizeof(float) * HW);
+    int32_t* owner = (int32_t*)malloc(sizeof(int32_t) * HW);
+    if (!depth || !owner) { free(depth); free(owner); return -2; }
+    for (size_t p = 0; p < HW; ++p) { depth[p] = INFINITY; owner[p] = -1; }
+    for (int f = 0; f < nf; ++f) {
+        float P[3][3], u[3], v[3];
+        int ok = 1;
+        for (int k = 0; k < 3; ++k) {
+            const int32_t vi = F[3 * (size_t)f + k];
+            if (vi < 0 || vi >= nv) { ok = 0; break; }
+            raster_cam_point(&c, V + 3 * (size_t)vi, P[k]);
+            if (!(P[k][2] > 1e-6f)) { ok = 0; break; }
+            u[k] = c.fx * (P[k][0] / P[k][2]) + c.cx;
+            v[k] = c.fy * (P[k][1] / P[k][2]) + c.cy;
+        }
+        if (!ok) continue;
+        const float area = (u[1] - u[0]) * (v[2] - v[0]) - (v[1] - v[0]) * (u[2] - u[0]);
+        if (!(area > 0.0f || area < 0.0f)) continue;
+        const float umin = fminf(u[0], fminf(u[1], u[2])), umax = fmaxf(u[0], fmaxf(u[1], u[2]));
+        const float vmin = fminf(v[0], fminf(v[1], v[2])), vmax = fmaxf(v[0], fmaxf(v[1], v[2]));
+        const float ilo = fmaxf(ceilf(umin - 0.5f), 0.0f), ihi = fminf(floorf(umax - 0.5f), (float)(W - 1));
+        const float jlo = fmaxf(ceilf(vmin - 0.5f), 0.0f), jhi = fminf(floorf(vmax - 0.5f), (float)(H - 1));
+        if (!(ilo <= ihi && jlo <= jhi)) continue;
+        float e1[3], e2[3], n[3];
+        for (int r = 0; r < 3; ++r) { e1[r] = P[1][r] - P[0][r]; e2[r] = P[2][r] - P[0][r]; }
+        n[0] = e1[1] * e2[2] - e1[2] * e2[1];
+        n[1] = e1[2] * e2[0] - e1[0] * e2[2];
+        n[2] = e1[0] * e2[1] - e1[1] * e2[0];
+        float nd = n[0] * P[0][0];
+        nd = nd + n[1] * P[0][1];
+        nd = nd + n[2] * P[0][2];
+        for (int j = (int)jlo; j <= (int)jhi; ++j) {
+            const float pv = (float)j + 0.5f;
+            for (int i = (int)ilo; i <= (int)ihi; ++i) {
+                const float pu = (float)i + 0.5f;
+                const float w0 = (u[2] - u[1]) * (pv - v[1]) - (v[2] - v[1]) * (pu - u[1]);
+                const float w1 = (u[0] - u[2]) * (pv - v[2]) - (v[0] - v[2]) * (pu - u[2]);
+                const float w2 = (u[1] - u[0]) * (pv - v[0]) - (v[1] - v[0]) * (pu - u[0]);
+                const int in = area > 0.0f ? (w0 >= 0.0f && w1 >= 0.0f && w2 >= 0.0f)
+                                           : (w0 <= 0.0f && w1 <= 0.0f && w2 <= 0.0f);
+                if (!in) continue;
+                float d[3];
+                const float s = raster_depth(&c, n, nd, pu, pv, d);
+                if (s == 0.0f) continue;
+                const size_t p = (size_t)j * W + i;
+                if (s < depth[p] || (s == depth[p] && f < owner[p])) { depth[p] = s; owner[p] = f; }
+            }
+        }
+    }
+    for (size_t p = 0; p < HW; ++p) {
+        float* X = pos_out + 3 * p;
+        X[0] = X[1] = X[2] = 0.0f;
+        valid_out[p] = owner[p] >= 0;
+        if (owner[p] < 0) continue;
+        /* the winner's plane and ray again, then world = R^T (x_c - t) */
+        const int f = owner[p];
+        float P[3][3], e1[3], e2[3], n[3], d[3];
+        for (int k = 0; k < 3; ++k) raster_cam_point(&c, V + 3 * (size_t)F[3 * (size_t)f + k], P[k]);
+        for (int r = 0; r < 3; ++r) { e1[r] = P[1][r] - P[0][r]; e2[r] = P[2][r] - P[0][r]; }
+        n[0] = e1[1] * e2[2] - e1[2] * e2[1];
+        n[1] = e1[2] * e2[0] - e1[0] * e2[2];
+        n[2] = e1[0] * e2[1] - e1[1] * e2[0];
+        float nd = n[0] * P[0][0];
+        nd = nd + n[1] * P[0][1];
+        nd = nd + n[2] * P[0][2];
+        const float s = raster_depth(&c, n, nd, (float)(p % W) + 0.5f, (float)(p / W) + 0.5f, d);
+        const float xc[3] = {s * d[0] - c.t[0], s * d[1] - c.t[1], s - c.t[2]};
+        for (int r = 0; r < 3; ++r) {
+            float x = c.R[r] * xc[0];
+            x = x + c.R[3 + r] * xc[1];
+            X[r] = x + c.R[6 + r] * xc[2];
+        }
+    }
+    free(depth);
+    free(owner);
+    return 0;
+}
