@@ -45,6 +45,7 @@ def parse():
     p.add_argument("--corr", default="sparse", choices=["sparse", "mask", "geometry", "table"])
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--no-raster", action="store_true", help="skip the position-map rasteriser measurement")
     p.add_argument("--cpu-assets", type=int, default=4, help="assets in the oracle's timed sample")
     return p.parse_args()
 
@@ -142,6 +143,53 @@ def measure_ablations(traj, reps=24):
     out["what"] = ("one cached step, %d assets, anchors %s, %d steps per graph; value_copy reads no anchor "
                    "x0(t-1); shuffled = records permuted within each (b, v, u) pair (seed 1)" % (w.B, anchors, reps))
     return out
+
+
+def measure_raster(dev, B, N_layout, H, W, reps=10, cpu_assets=2):
+    """Position maps of B meshes (icosphere subdivision 6 with smooth radial
+    noise: 40962 vertices, 81920 faces; four distinct meshes tiled over the
+    batch) seen by the workload's N cameras (azimuths offset per asset), at
+    H x W: GPU time of one geocache_raster_posmaps call (z-buffer clear,
+    face kernel, resolve kernel) and the oracle's single-threaded time on
+    `cpu_assets` of the assets."""
+    import torch
+    import oracle
+    from paper_2608_13255_gb300 import geocache as gc
+    from paper_2608_13255_gb300 import synth
+    base = [synth.blob_mesh(6, 0.15, np.random.default_rng(100 + k)) for k in range(4)]
+    meshes = [(base[b % 4][0].astype(np.float32), base[b % 4][1].astype(np.int32)) for b in range(B)]
+    cams = np.stack([np.stack([synth.look_at_camera(az + 7.0 * b, el, H, W) for az, el in N_layout])
+                     for b in range(B)])
+    v_off = np.cumsum([0] + [len(V) for V, _ in meshes])
+    f_off = torch.from_numpy(np.cumsum([0] + [len(F) for _, F in meshes]).astype(np.int64)).to(dev)
+    verts = torch.from_numpy(np.concatenate([V for V, _ in meshes])).to(dev)
+    faces = torch.from_numpy(np.concatenate([F + v_off[b] for b, (_, F) in enumerate(meshes)]).astype(np.int32)).to(dev)
+    d_cams = torch.from_numpy(cams).to(dev)
+    N = len(N_layout)
+    zbuf = torch.empty((B, N, H, W), dtype=torch.int64, device=dev)
+    pos = torch.empty((B, N, H, W, 3), dtype=torch.float32, device=dev)
+    valid = torch.empty((B, N, H, W), dtype=torch.uint8, device=dev)
+    for _ in range(2):
+        gc.raster_posmaps(verts, faces, f_off, d_cams, H, W, zbuf, pos, valid)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(reps):
+        gc.raster_posmaps(verts, faces, f_off, d_cams, H, W, zbuf, pos, valid)
+    e1.record()
+    torch.cuda.synchronize()
+    gc.device_status()
+    us = e0.elapsed_time(e1) * 1e3 / reps
+    pixels, face_views = B * N * H * W, N * int(faces.shape[0])
+    t0 = time.perf_counter()
+    for b in range(cpu_assets):
+        oracle.raster_views(meshes[b][0], meshes[b][1], cams[b], H, W)
+    cpu_s = time.perf_counter() - t0
+    return {"what": "%d meshes x %d views at %dx%d, 81920 faces each" % (B, N, H, W),
+            "us_per_batch": us, "pixels_per_s": pixels / us * 1e6, "face_views_per_s": face_views / us * 1e6,
+            "covered_frac": float(valid.float().mean()), "launches_per_call": 2,
+            "cpu_oracle": {"pixels_per_s": cpu_assets * N * H * W / cpu_s, "cores": 1,
+                           "sample": "%d of the meshes, all views" % cpu_assets}}
 
 
 class Trajectory:
@@ -551,6 +599,11 @@ def main():
         del srcs, sls
 
     ablations = measure_ablations(traj) if rank == 0 and args.corr == "sparse" else None
+    raster = None
+    if rank == 0 and not args.no_raster:
+        from paper_2608_13255_gb300 import synth
+        layout = synth.hunyuan_layout() if w.N == 6 else synth.ring8_polar4_layout()[:w.N]
+        raster = measure_raster(dev, w.B, layout, w.H, w.W)
 
     e2e = None
     if not args.no_e2e:
@@ -586,6 +639,7 @@ def main():
         "gpu_launches": launches,
         "pack_anchors": pack,
         "ablations": ablations,
+        "raster_posmaps": raster,
         "clocks": clocks.summary(),
         "e2e": e2e,
     }

@@ -273,6 +273,36 @@ int geocache_transport_step_update(const geocache_corr* corr, geocache_update up
 int geocache_permute_records(const geocache_corr* corr, const int32_t* perm, geocache_tap_record* out, void* stream);
 
 /* --------------------------------------------------------------------------
+ * geocache_raster_posmaps -- the position maps and validity masks of B
+ * triangle meshes, each seen by N cameras (the rendered position maps of
+ * Sec. 3.1 that the correspondence operator of Sec. 3.2 is built from), by a
+ * z-buffer over pixel centres: pixel (i, j) is covered by a face when its
+ * centre (i + 0.5, j + 0.5) lies inside or on the face's projection (faces
+ * with a vertex at camera z <= 1e-6 or zero projected area are skipped);
+ * the nearest such face along the pixel's ray wins (ties to the lower face
+ * index) and pos holds the world position of that ray / face-plane
+ * intersection.  Decisions and positions are binary32, one rounding per
+ * operation in a fixed order, so the maps are reproducible bit for bit.
+ *   verts     device [n_verts, 3] f32 world positions of all meshes.
+ *   faces     device [n_faces, 3] i32 indices into verts; faces of asset b
+ *             are faces[face_off[b] .. face_off[b+1]).  A face with an index
+ *             outside [0, n_verts) is skipped and reported in the device
+ *             status word (geocache_device_status then returns EINVAL).
+ *   face_off  device [B + 1] i64, ascending, face_off[0] = 0,
+ *             face_off[B] = n_faces (n_faces < 2^32).
+ *   cams      device [B, N] cameras (geocache_camera).
+ *   zbuf      device [B, N, H, W] u64 scratch (overwritten).
+ *   pos, valid  device [B, N, H, W, 3] f32 / [B, N, H, W] u8 outputs, the
+ *             layout of geocache_corr.pos / .valid; uncovered pixels get
+ *             position 0 and valid 0.
+ * Asynchronous.  Sizes: 1 <= B <= 65535, 1 <= N <= GEOCACHE_MAX_VIEWS,
+ * 1 <= H, W <= 16384.  Returns GEOCACHE_OK, EINVAL, ESHAPE, EALIAS, ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_raster_posmaps(const float* verts, int64_t n_verts, const int32_t* faces, int64_t n_faces,
+                            const int64_t* face_off, int B, const geocache_camera* cams, int N, int H, int W,
+                            uint64_t* zbuf, float* pos, uint8_t* valid, void* stream);
+
+/* --------------------------------------------------------------------------
  * geocache_reconstruct -- full-step passthrough (Sec. 3.2: at a full step the
  * denoiser runs on all N views and its x0 is both the new reference and the
  * input of the sampler conversion).
@@ -334,10 +364,11 @@ int geocache_rotate_anchors(int N, int a, int step, int S, const geocache_schedu
  * trapping, so the context stays usable: a sparse-form build whose records
  * exceed max_records (the excess is dropped; transport steps read only the
  * records that exist), a record permutation entry out of range
- * (geocache_permute_records keeps that record), and a bounded wait inside a
+ * (geocache_permute_records keeps that record), a mesh face with a vertex
+ * index out of range (geocache_raster_posmaps skips it), and a bounded wait inside a
  * kernel that ran out (its CTA returns without writing its outputs).
  * Returns GEOCACHE_OK, ESHAPE (record overflow), EINVAL (bad permutation
- * entry), ETIMEOUT (a wait gave up) or ECUDA.
+ * entry or face index), ETIMEOUT (a wait gave up) or ECUDA.
  * ------------------------------------------------------------------------ */
 int geocache_device_status(void* stream);
 

@@ -116,15 +116,20 @@ extern "C" {
 int geocache_abi_version(void) { return GEOCACHE_ABI_VERSION; }
 
 int geocache_device_status(void* stream) {
-    unsigned int word = 0;
+    unsigned int word = 0, raster_word = 0;
     cudaError_t e = geocache::read_device_error(&word, true, (cudaStream_t)stream);
+    if (e == cudaSuccess) e = geocache::read_raster_error(&raster_word, true, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "reading the device status word");
+    word |= raster_word;
     if (word & 2u)
         return fail(GEOCACHE_ESHAPE, "a sparse-form build had more records than max_records (status word 0x%x); "
                                      "query geocache_corr_record_count and rebuild", word);
     if (word & 4u)
         return fail(GEOCACHE_EINVAL, "a record permutation entry was outside [0, max_records) (status word 0x%x); "
                                      "those records were kept", word);
+    if (word & 8u)
+        return fail(GEOCACHE_EINVAL, "a mesh face had a vertex index outside [0, n_verts) (status word 0x%x); "
+                                     "those faces were skipped", word);
     if (word) return fail(GEOCACHE_ETIMEOUT, "a bounded device wait gave up (status word 0x%x); outputs of that call are incomplete", word);
     return ok();
 }
@@ -319,6 +324,34 @@ int geocache_permute_records(const geocache_corr* c, const int32_t* perm, geocac
         return fail(GEOCACHE_EALIAS, "out overlaps the records or the permutation");
     cudaError_t e = geocache::launch_permute_records(c->records, perm, out, c->max_records, (cudaStream_t)stream);
     if (e != cudaSuccess) return cuda_fail(e, "record permutation kernel launch");
+    return ok();
+}
+
+int geocache_raster_posmaps(const float* verts, int64_t n_verts, const int32_t* faces, int64_t n_faces,
+                            const int64_t* face_off, int B, const geocache_camera* cams, int N, int H, int W,
+                            uint64_t* zbuf, float* pos, uint8_t* valid, void* stream) {
+    if (B < 1 || B > 65535 || N < 1 || N > GEOCACHE_MAX_VIEWS || H < 1 || W < 1 || H > 16384 || W > 16384)
+        return fail(GEOCACHE_ESHAPE, "B=%d, N=%d, H=%d, W=%d out of range", B, N, H, W);
+    if (n_verts < 0 || n_faces < 0 || n_faces > 0xffffffffLL || n_verts > 0x7fffffffLL)
+        return fail(GEOCACHE_ESHAPE, "n_verts=%lld, n_faces=%lld out of range", (long long)n_verts, (long long)n_faces);
+    if (!cams || !face_off || !zbuf || !pos || !valid || (n_faces > 0 && (!verts || !faces)))
+        return fail(GEOCACHE_EINVAL, "verts, faces, face_off, cams, zbuf, pos and valid are required");
+    if ((uintptr_t)zbuf & 7) return fail(GEOCACHE_EINVAL, "zbuf must be 8-byte aligned");
+    const size_t px = (size_t)B * N * H * W;
+    const void* outs[3] = {zbuf, pos, valid};
+    const size_t ob[3] = {px * 8, px * 12, px};
+    const void* ins[5] = {verts, faces, face_off, cams, nullptr};
+    const size_t ib[5] = {(size_t)n_verts * 12, (size_t)n_faces * 12, (size_t)(B + 1) * 8, sizeof(geocache_camera) * B * N, 0};
+    for (int i = 0; i < 3; ++i) {
+        for (int j = i + 1; j < 3; ++j)
+            if (overlap(outs[i], ob[i], outs[j], ob[j])) return fail(GEOCACHE_EALIAS, "zbuf, pos and valid overlap");
+        for (int j = 0; j < 4; ++j)
+            if (overlap(outs[i], ob[i], ins[j], ib[j])) return fail(GEOCACHE_EALIAS, "an output overlaps an input");
+    }
+    cudaError_t e = geocache::launch_raster(verts, n_verts, faces, n_faces, face_off, B, cams, N, H, W,
+                                            reinterpret_cast<unsigned long long*>(zbuf), pos, valid,
+                                            (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "rasteriser launch");
     return ok();
 }
 

@@ -71,6 +71,10 @@ cudaError_t launch_reconstruct(const void* x_t, const float* x0, void* x_next, i
                                const ReconCoef& coef, float* pred_out, float* x0_store, cudaStream_t s);
 
 cudaError_t read_device_error(unsigned int* out, bool clear, cudaStream_t s);
+cudaError_t read_raster_error(unsigned int* out, bool clear, cudaStream_t s);
+cudaError_t launch_raster(const float* V, long long nv, const int32_t* F, long long nf, const int64_t* face_off,
+                          int B, const geocache_camera* cams, int N, int H, int W, unsigned long long* zbuf,
+                          float* pos, uint8_t* valid, cudaStream_t s);
 
 // Records a status and its message for geocache_last_error(); returns status.
 int set_error(int status, const char* fmt, ...);

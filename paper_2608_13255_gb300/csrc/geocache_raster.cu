@@ -1,0 +1,288 @@
+// Position-map rasteriser: the per-pixel world positions and validity masks
+// that a geometry-conditioned texturing pipeline renders for each view
+// (Sec. 3.1), from which the correspondence operator of Sec. 3.2 is built.
+//
+// A z-buffer over pixel centres, in two kernels:
+//  raster_faces_kernel: one thread per (face, view).  The face is projected;
+//    every pixel centre inside or on it (three sign-normalised edge
+//    functions) gets the camera z of the ray / face-plane intersection, and
+//    the key (depth bits << 32 | face index) is min-combined into the
+//    pixel's z-buffer word with a 64-bit atomicMin (nearest face wins, ties
+//    to the lower face index; positive floats order like their bits).  A
+//    face whose pixel box exceeds kSmallBox pixels is handed to its whole
+//    warp, whose 32 lanes stride over the box, so that a few large faces do
+//    not serialise on one thread.
+//  raster_resolve_kernel: one thread per pixel; the key's depth gives the
+//    world position of the intersection.
+// Every decision and the position are binary32 with one rounding per
+// operation in a fixed order (explicit __f*_rn intrinsics), so the maps are
+// reproducible bit for bit.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "geocache.h"
+#include "geocache_internal.h"
+
+namespace geocache {
+
+namespace {
+
+// Status word of this translation unit (the library is linked without
+// relocatable device code): bit 3 = a face index outside [0, nv).  Read and
+// cleared together with the transport's word by geocache_device_status.
+__device__ unsigned int g_raster_error = 0;
+
+constexpr int kRasterThreads = 256;
+constexpr int kSmallBox = 64;                 // pixels a single thread rasterises
+constexpr unsigned long long kEmpty = ~0ull;  // z-buffer word of an uncovered pixel
+
+struct Cam32 {
+    float R[9], t[3], fx, fy, cx, cy;
+};
+
+__device__ __forceinline__ Cam32 load_cam(const geocache_camera* c) {
+    Cam32 k;
+    const float* p = reinterpret_cast<const float*>(c);
+#pragma unroll
+    for (int i = 0; i < 9; ++i) k.R[i] = __ldg(p + i);
+#pragma unroll
+    for (int i = 0; i < 3; ++i) k.t[i] = __ldg(p + 9 + i);
+    k.fx = __ldg(p + 12);
+    k.fy = __ldg(p + 13);
+    k.cx = __ldg(p + 14);
+    k.cy = __ldg(p + 15);
+    return k;
+}
+
+// x_c = R X + t, each row summed ((R0 X0 + R1 X1) + R2 X2) + t
+__device__ __forceinline__ void cam_point(const Cam32& c, const float* X, float* xc) {
+#pragma unroll
+    for (int r = 0; r < 3; ++r) {
+        float s = __fmul_rn(c.R[3 * r], __ldg(X));
+        s = __fadd_rn(s, __fmul_rn(c.R[3 * r + 1], __ldg(X + 1)));
+        s = __fadd_rn(s, __fmul_rn(c.R[3 * r + 2], __ldg(X + 2)));
+        xc[r] = __fadd_rn(s, c.t[r]);
+    }
+}
+
+// One projected face: screen vertices, signed area, camera-space plane
+// n . x = nd, and the clamped pixel box.
+struct Face {
+    float u[3], v[3], area, n[3], nd;
+    int ilo, ihi, jlo, jhi;
+};
+
+// false when the face covers no pixel centre: an index outside [0, nv)
+// (reported in the status word), a vertex not in front (z <= 1e-6), zero
+// area, or a box outside the image
+__device__ __forceinline__ bool setup_face(const Cam32& c, const float* __restrict__ V, long long nv,
+                                           const int32_t* __restrict__ F, long long f, int H, int W, Face& o) {
+    float P[3][3];
+#pragma unroll
+    for (int k = 0; k < 3; ++k) {
+        const int32_t vi = __ldg(F + 3 * f + k);
+        if (vi < 0 || vi >= nv) {
+            atomicOr(&g_raster_error, 8u);
+            return false;
+        }
+        cam_point(c, V + 3 * (size_t)vi, P[k]);
+        if (!(P[k][2] > 1e-6f)) return false;
+        o.u[k] = __fadd_rn(__fmul_rn(c.fx, __fdiv_rn(P[k][0], P[k][2])), c.cx);
+        o.v[k] = __fadd_rn(__fmul_rn(c.fy, __fdiv_rn(P[k][1], P[k][2])), c.cy);
+    }
+    o.area = __fsub_rn(__fmul_rn(__fsub_rn(o.u[1], o.u[0]), __fsub_rn(o.v[2], o.v[0])),
+                       __fmul_rn(__fsub_rn(o.v[1], o.v[0]), __fsub_rn(o.u[2], o.u[0])));
+    if (!(o.area > 0.0f || o.area < 0.0f)) return false;
+    const float umin = fminf(o.u[0], fminf(o.u[1], o.u[2])), umax = fmaxf(o.u[0], fmaxf(o.u[1], o.u[2]));
+    const float vmin = fminf(o.v[0], fminf(o.v[1], o.v[2])), vmax = fmaxf(o.v[0], fmaxf(o.v[1], o.v[2]));
+    const float ilo = fmaxf(ceilf(__fsub_rn(umin, 0.5f)), 0.0f), ihi = fminf(floorf(__fsub_rn(umax, 0.5f)), (float)(W - 1));
+    const float jlo = fmaxf(ceilf(__fsub_rn(vmin, 0.5f)), 0.0f), jhi = fminf(floorf(__fsub_rn(vmax, 0.5f)), (float)(H - 1));
+    if (!(ilo <= ihi && jlo <= jhi)) return false;
+    o.ilo = (int)ilo;
+    o.ihi = (int)ihi;
+    o.jlo = (int)jlo;
+    o.jhi = (int)jhi;
+    float e1[3], e2[3];
+#pragma unroll
+    for (int r = 0; r < 3; ++r) {
+        e1[r] = __fsub_rn(P[1][r], P[0][r]);
+        e2[r] = __fsub_rn(P[2][r], P[0][r]);
+    }
+    o.n[0] = __fsub_rn(__fmul_rn(e1[1], e2[2]), __fmul_rn(e1[2], e2[1]));
+    o.n[1] = __fsub_rn(__fmul_rn(e1[2], e2[0]), __fmul_rn(e1[0], e2[2]));
+    o.n[2] = __fsub_rn(__fmul_rn(e1[0], e2[1]), __fmul_rn(e1[1], e2[0]));
+    float nd = __fmul_rn(o.n[0], P[0][0]);
+    nd = __fadd_rn(nd, __fmul_rn(o.n[1], P[0][1]));
+    o.nd = __fadd_rn(nd, __fmul_rn(o.n[2], P[0][2]));
+    return true;
+}
+
+// camera-space ray direction through the pixel centre (pu, pv)
+__device__ __forceinline__ void ray(const Cam32& c, float pu, float pv, float& d0, float& d1) {
+    d0 = __fdiv_rn(__fsub_rn(pu, c.cx), c.fx);
+    d1 = __fdiv_rn(__fsub_rn(pv, c.cy), c.fy);
+}
+
+// depth key of pixel (i, j) for the face, or kEmpty when its centre is not
+// covered or the ray meets the plane at no positive finite depth
+__device__ __forceinline__ unsigned long long pixel_key(const Cam32& c, const Face& o, int i, int j,
+                                                        unsigned int face) {
+    const float pu = __fadd_rn((float)i, 0.5f), pv = __fadd_rn((float)j, 0.5f);
+    const float w0 = __fsub_rn(__fmul_rn(__fsub_rn(o.u[2], o.u[1]), __fsub_rn(pv, o.v[1])),
+                               __fmul_rn(__fsub_rn(o.v[2], o.v[1]), __fsub_rn(pu, o.u[1])));
+    const float w1 = __fsub_rn(__fmul_rn(__fsub_rn(o.u[0], o.u[2]), __fsub_rn(pv, o.v[2])),
+                               __fmul_rn(__fsub_rn(o.v[0], o.v[2]), __fsub_rn(pu, o.u[2])));
+    const float w2 = __fsub_rn(__fmul_rn(__fsub_rn(o.u[1], o.u[0]), __fsub_rn(pv, o.v[0])),
+                               __fmul_rn(__fsub_rn(o.v[1], o.v[0]), __fsub_rn(pu, o.u[0])));
+    const bool in = o.area > 0.0f ? (w0 >= 0.0f && w1 >= 0.0f && w2 >= 0.0f)
+                                  : (w0 <= 0.0f && w1 <= 0.0f && w2 <= 0.0f);
+    if (!in) return kEmpty;
+    float d0, d1;
+    ray(c, pu, pv, d0, d1);
+    float den = __fmul_rn(o.n[0], d0);
+    den = __fadd_rn(den, __fmul_rn(o.n[1], d1));
+    den = __fadd_rn(den, o.n[2]);
+    if (den == 0.0f) return kEmpty;
+    const float s = __fdiv_rn(o.nd, den);
+    if (!(s > 0.0f && s <= 3.0e38f)) return kEmpty;
+    return ((unsigned long long)__float_as_uint(s) << 32) | face;
+}
+
+// asset of face f: face_off[b] <= f < face_off[b + 1] (clamped to [0, B))
+__device__ __forceinline__ int asset_of(const int64_t* __restrict__ face_off, int B, long long f) {
+    int lo = 0, hi = B - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (__ldg(face_off + mid) <= f) lo = mid;
+        else hi = mid - 1;
+    }
+    return lo;
+}
+
+__global__ void __launch_bounds__(kRasterThreads) raster_faces_kernel(
+    const float* __restrict__ V, long long nv, const int32_t* __restrict__ F, long long nf,
+    const int64_t* __restrict__ face_off, int B, const geocache_camera* __restrict__ cams, int N, int H, int W,
+    unsigned long long* __restrict__ zbuf) {
+    const long long f = blockIdx.x * (long long)kRasterThreads + threadIdx.x;
+    const int view = blockIdx.y;
+    const int lane = threadIdx.x & 31;
+    Face o;
+    Cam32 c;
+    bool live = false;
+    int b = 0;
+    if (f < nf) {
+        b = asset_of(face_off, B, f);
+        c = load_cam(cams + (size_t)b * N + view);
+        live = setup_face(c, V, nv, F, f, H, W, o);
+    }
+    const long long box = live ? (long long)(o.ihi - o.ilo + 1) * (o.jhi - o.jlo + 1) : 0;
+    unsigned long long* zb = zbuf + ((size_t)b * N + view) * (size_t)H * W;
+    if (live && box <= kSmallBox) {
+        for (int j = o.jlo; j <= o.jhi; ++j)
+            for (int i = o.ilo; i <= o.ihi; ++i) {
+                const unsigned long long key = pixel_key(c, o, i, j, (unsigned int)f);
+                if (key != kEmpty) atomicMin(zb + (size_t)j * W + i, key);
+            }
+    }
+    // large faces: the warp takes them one at a time
+    unsigned big = __ballot_sync(0xffffffffu, live && box > kSmallBox);
+    while (big) {
+        const int src = __ffs(big) - 1;
+        big &= big - 1;
+        Face q;
+#pragma unroll
+        for (int k = 0; k < 3; ++k) {
+            q.u[k] = __shfl_sync(0xffffffffu, o.u[k], src);
+            q.v[k] = __shfl_sync(0xffffffffu, o.v[k], src);
+            q.n[k] = __shfl_sync(0xffffffffu, o.n[k], src);
+        }
+        q.area = __shfl_sync(0xffffffffu, o.area, src);
+        q.nd = __shfl_sync(0xffffffffu, o.nd, src);
+        q.ilo = __shfl_sync(0xffffffffu, o.ilo, src);
+        q.ihi = __shfl_sync(0xffffffffu, o.ihi, src);
+        q.jlo = __shfl_sync(0xffffffffu, o.jlo, src);
+        q.jhi = __shfl_sync(0xffffffffu, o.jhi, src);
+        const int qb = __shfl_sync(0xffffffffu, b, src);
+        const long long qf = __shfl_sync(0xffffffffu, f, src);
+        const Cam32 qc = load_cam(cams + (size_t)qb * N + view);
+        unsigned long long* qz = zbuf + ((size_t)qb * N + view) * (size_t)H * W;
+        const int bw = q.ihi - q.ilo + 1;
+        const long long n = (long long)bw * (q.jhi - q.jlo + 1);
+        for (long long k = lane; k < n; k += 32) {
+            const int i = q.ilo + (int)(k % bw), j = q.jlo + (int)(k / bw);
+            const unsigned long long key = pixel_key(qc, q, i, j, (unsigned int)qf);
+            if (key != kEmpty) atomicMin(qz + (size_t)j * W + i, key);
+        }
+    }
+}
+
+__global__ void __launch_bounds__(kRasterThreads) raster_resolve_kernel(const unsigned long long* __restrict__ zbuf,
+                                                                         const geocache_camera* __restrict__ cams,
+                                                                         int N, int H, int W, long long n_pix,
+                                                                         float* __restrict__ pos,
+                                                                         uint8_t* __restrict__ valid) {
+    const long long HW = (long long)H * W;
+    for (long long p = blockIdx.x * (long long)kRasterThreads + threadIdx.x; p < n_pix;
+         p += (long long)gridDim.x * kRasterThreads) {
+        const unsigned long long key = zbuf[p];
+        float X[3] = {0.0f, 0.0f, 0.0f};
+        if (key != kEmpty) {
+            const Cam32 c = load_cam(cams + p / HW);  // [B, N] cameras, one per (asset, view) map
+            const int pix = (int)(p % HW);
+            const float s = __uint_as_float((unsigned int)(key >> 32));
+            float d0, d1;
+            ray(c, __fadd_rn((float)(pix % W), 0.5f), __fadd_rn((float)(pix / W), 0.5f), d0, d1);
+            const float xc[3] = {__fsub_rn(__fmul_rn(s, d0), c.t[0]), __fsub_rn(__fmul_rn(s, d1), c.t[1]),
+                                 __fsub_rn(s, c.t[2])};
+#pragma unroll
+            for (int r = 0; r < 3; ++r) {
+                float x = __fmul_rn(c.R[r], xc[0]);
+                x = __fadd_rn(x, __fmul_rn(c.R[3 + r], xc[1]));
+                X[r] = __fadd_rn(x, __fmul_rn(c.R[6 + r], xc[2]));
+            }
+        }
+        pos[3 * p] = X[0];
+        pos[3 * p + 1] = X[1];
+        pos[3 * p + 2] = X[2];
+        valid[p] = key != kEmpty;
+    }
+}
+
+}  // namespace
+
+cudaError_t read_raster_error(unsigned int* out, bool clear, cudaStream_t s) {
+    cudaError_t e = cudaMemcpyFromSymbolAsync(out, g_raster_error, sizeof(unsigned int), 0, cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return e;
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess || !clear || *out == 0) return e;
+    static const unsigned int zero = 0;
+    e = cudaMemcpyToSymbolAsync(g_raster_error, &zero, sizeof(unsigned int), 0, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return e;
+    return cudaStreamSynchronize(s);
+}
+
+cudaError_t launch_raster(const float* V, long long nv, const int32_t* F, long long nf, const int64_t* face_off,
+                          int B, const geocache_camera* cams, int N, int H, int W, unsigned long long* zbuf,
+                          float* pos, uint8_t* valid, cudaStream_t s) {
+    const long long n_pix = (long long)B * N * H * W;
+    cudaError_t e = cudaMemsetAsync(zbuf, 0xff, sizeof(unsigned long long) * (size_t)n_pix, s);
+    if (e != cudaSuccess) return e;
+    if (nf > 0) {
+        const long long gx = (nf + kRasterThreads - 1) / kRasterThreads;
+        if (gx > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+        raster_faces_kernel<<<dim3((unsigned)gx, N), kRasterThreads, 0, s>>>(V, nv, F, nf, face_off, B, cams, N, H,
+                                                                              W, zbuf);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const long long want = (n_pix + kRasterThreads - 1) / kRasterThreads, cap = (long long)(sms > 0 ? sms : 1) * 16;
+    raster_resolve_kernel<<<(unsigned)(want < cap ? (want > 0 ? want : 1) : cap), kRasterThreads, 0, s>>>(
+        zbuf, cams, N, H, W, n_pix, pos, valid);
+    return cudaGetLastError();
+}
+
+}  // namespace geocache

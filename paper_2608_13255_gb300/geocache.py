@@ -70,6 +70,7 @@ EXPORTS = ("geocache_build_corr", "geocache_transport_step", "geocache_reconstru
            "geocache_rotate_anchors", "geocache_device_status", "geocache_corr_record_count",
            "geocache_transport_workspace", "geocache_transport_step_noalloc", "geocache_pack_anchors",
            "geocache_unpack_anchors", "geocache_transport_step_update", "geocache_permute_records",
+           "geocache_raster_posmaps",
            "geocache_last_error", "geocache_abi_version")
 
 
@@ -98,6 +99,8 @@ def load():
         L.geocache_transport_step_update.restype = ctypes.c_int
         L.geocache_permute_records.argtypes = [ctypes.POINTER(Corr), P, P, P]
         L.geocache_permute_records.restype = ctypes.c_int
+        L.geocache_raster_posmaps.argtypes = [P, i64, P, i64, P, i, P, i, i, i, P, P, P, P]
+        L.geocache_raster_posmaps.restype = ctypes.c_int
         for name in ("geocache_pack_anchors", "geocache_unpack_anchors"):
             getattr(L, name).argtypes = [P, P, i64, i, i, P, i, P]
             getattr(L, name).restype = ctypes.c_int
@@ -328,6 +331,30 @@ def permute_records(corr: CorrHandle, perm, out=None, stream=None) -> CorrHandle
     c2.records = out.data_ptr()
     c2.mode = CORR_SPARSE
     return CorrHandle(c2, refs)
+
+
+def raster_posmaps(verts, faces, face_off, cams, H, W, zbuf=None, pos=None, valid=None, stream=None):
+    """geocache_raster_posmaps: position maps [B,N,H,W,3] f32 and validity
+    [B,N,H,W] u8 of B meshes (verts [V,3] f32, faces [F,3] i32 indexing
+    verts, face_off [B+1] i64, all on the device) seen by cams [B,N,16].
+    Returns (pos, valid); zbuf is the [B,N,H,W] int64 scratch."""
+    B, N = int(cams.shape[0]), int(cams.shape[1])
+    dev = cams.device
+    if zbuf is None:
+        zbuf = torch.empty((B, N, H, W), dtype=torch.int64, device=dev)
+    if pos is None:
+        pos = torch.empty((B, N, H, W, 3), dtype=torch.float32, device=dev)
+    if valid is None:
+        valid = torch.empty((B, N, H, W), dtype=torch.uint8, device=dev)
+    nv, nf = int(verts.shape[0]), int(faces.shape[0])
+    n = B * N * H * W
+    _check(load().geocache_raster_posmaps(
+        _dev(verts, torch.float32, 3 * nv, "verts") if nv else None, nv,
+        _dev(faces, torch.int32, 3 * nf, "faces") if nf else None, nf,
+        _dev(face_off, torch.int64, B + 1, "face_off"), B, _dev(cams, torch.float32, 16 * B * N, "cams"), N,
+        int(H), int(W), _dev(zbuf, torch.int64, n, "zbuf"), _dev(pos, torch.float32, 3 * n, "pos"),
+        _dev(valid, torch.uint8, n, "valid"), _stream(stream)))
+    return pos, valid
 
 
 def transport_step_noalloc(corr: CorrHandle, anchors, C, x0_anchor_new, x0_prev, x0_out, x_t=None, x_next=None,

@@ -147,3 +147,19 @@ def test_ablation_entry_points_check_arguments(gc):
     c.records, c.max_records = 4096, 64
     assert L.geocache_permute_records(ctypes.byref(c), 16, 4096 + 512, None) == gc.EALIAS  # out overlaps records
     assert L.geocache_permute_records(ctypes.byref(c), 16, 4100, None) == gc.EINVAL  # misaligned out
+
+
+def test_raster_entry_point_checks_arguments(gc):
+    L = gc.load()
+    P = 4096
+    # sizes
+    assert L.geocache_raster_posmaps(P, 3, P, 1, P, 0, P, 6, 8, 8, P, P, P, None) == gc.ESHAPE
+    assert L.geocache_raster_posmaps(P, 3, P, 1, P, 1, P, 65, 8, 8, P, P, P, None) == gc.ESHAPE
+    assert L.geocache_raster_posmaps(P, -1, P, 1, P, 1, P, 6, 8, 8, P, P, P, None) == gc.ESHAPE
+    # required buffers, alignment, overlaps
+    assert L.geocache_raster_posmaps(None, 3, P, 1, P, 1, P, 6, 8, 8, P, P, P, None) == gc.EINVAL
+    assert L.geocache_raster_posmaps(P, 3, P, 1, P, 1, P, 6, 8, 8, P + 4, 1 << 20, 1 << 21, None) == gc.EINVAL
+    st = L.geocache_raster_posmaps(1 << 24, 3, 1 << 25, 1, 1 << 26, 1, 1 << 27, 6, 8, 8, 1 << 20, 1 << 20, 1 << 22, None)
+    assert st == gc.EALIAS and "overlap" in gc.last_error()
+    st = L.geocache_raster_posmaps(1 << 20, 3, 1 << 25, 1, 1 << 26, 1, 1 << 27, 6, 8, 8, 1 << 20, 1 << 21, 1 << 22, None)
+    assert st == gc.EALIAS  # zbuf over the vertices
