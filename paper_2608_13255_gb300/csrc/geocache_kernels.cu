@@ -257,12 +257,12 @@ __device__ __forceinline__ int tiles_per_view_dev(int H, int W) {
 __global__ void __launch_bounds__(1024) exclusive_scan_kernel(int32_t* a, long long n) {
     __shared__ long long s_warp[32];
     __shared__ long long s_carry;
-    constexpr int kItems = 8;
+    constexpr int kItems = 16;
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
     if (t == 0) s_carry = 0;
     __syncthreads();
     for (long long base = 0; base < n; base += 1024LL * kItems) {
-        long long v[kItems];
+        int v[kItems];
         long long sum = 0;
 #pragma unroll
         for (int i = 0; i < kItems; ++i) {
@@ -299,7 +299,10 @@ __global__ void __launch_bounds__(1024) exclusive_scan_kernel(int32_t* a, long l
         if (t == 0) s_carry += s_warp[31];
         __syncthreads();
     }
-    if (t == 0) a[n] = s_carry > 0x7fffffffLL ? -1 : (int32_t)s_carry;
+    if (t == 0) {
+        a[n] = s_carry > 0x7fffffffLL ? -1 : (int32_t)s_carry;
+        if (s_carry > 0x7fffffffLL) atomicOr(&g_device_error, 2u);  // more records than int32 offsets index
+    }
 }
 
 // tile_ptr holds the per-tile counts written by build_corr_kernel; turn them
@@ -324,6 +327,11 @@ __global__ void __launch_bounds__(256) fill_records_kernel(const float* __restri
     const int v = vu / N, u = vu % N;
     const int HW = H * W;
     const int t = threadIdx.x;
+    // the tile's first record; a tile without records (and every diagonal
+    // pair) has nothing to write
+    const size_t ti = ((size_t)b * N * N + vu) * T + tile;
+    const int r_first = __ldg(tile_ptr + ti);
+    if (u == v || __ldg(tile_ptr + ti + 1) == r_first || r_first < 0) return;  // < 0: offsets overflowed (flagged)
     __shared__ geocache_camera s_cam;
     __shared__ int s_warp[8];
     if (t < 16) reinterpret_cast<float*>(&s_cam)[t] = __ldg(reinterpret_cast<const float*>(cams + (size_t)b * N + u) + t);
@@ -349,7 +357,7 @@ __global__ void __launch_bounds__(256) fill_records_kernel(const float* __restri
     __syncthreads();
     int base = 0;
     for (int w = 0; w < warp; ++w) base += s_warp[w];
-    long long r = (long long)__ldg(tile_ptr + ((size_t)b * N * N + vu) * T + tile) + base + incl - mine;
+    long long r = (long long)r_first + base + incl - mine;
     const size_t tv0 = ((size_t)b * N + v) * HW;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -1045,6 +1053,15 @@ __device__ __forceinline__ int nonanchor_view(const TransportArgs& args, int vi)
     return -1;
 }
 
+// Tile offset i of the sparse form clamped to the records that exist, [0,
+// cap]: a build whose records overflowed the capacity or the int32 offsets
+// is flagged in the status word, and the transport then reads only records
+// that exist.
+__device__ __forceinline__ int record_offset(const int32_t* __restrict__ tile_ptr, size_t i, long long cap) {
+    const long long x = __ldg(tile_ptr + i);
+    return (int)(x < 0 ? 0 : (x < cap ? x : cap));
+}
+
 // Records of one pair applied by one CTA slice (grid-stride over the pair's records).
 // COPY: the value-copy ablation (no x0(t-1) gathers).
 template <int K, bool COPY>
@@ -1059,8 +1076,8 @@ __device__ __forceinline__ void apply_records(const TransportArgs& args, int pai
     const int u = args.anchors[s2];
     const size_t pair = ((size_t)b * N + v) * N + u;
     const long long cap = args.max_records;
-    const int r0 = (int)min((long long)__ldg(args.tile_ptr + pair * T), cap);
-    const int r1 = (int)min((long long)__ldg(args.tile_ptr + pair * T + T), cap);
+    const int r0 = record_offset(args.tile_ptr, pair * T, cap);
+    const int r1 = record_offset(args.tile_ptr, pair * T + T, cap);
     const size_t plane = (size_t)HW;
     const float* xn = args.x0_new + ((size_t)b * a + s2) * C * plane;
     const float* xp = args.x0_prev + ((size_t)b * N + u) * C * plane;
@@ -1173,9 +1190,9 @@ __global__ void __launch_bounds__(kThreads) sparse_phase_b_kernel(const Transpor
     if (t < a) {
         const size_t i = (((size_t)b * N + v) * N + args.anchors[t]) * T_tiles + tile;
         // ranges clamped to the records that exist (an overflow is reported by the build)
-        const int r0 = (int)min((long long)__ldg(args.tile_ptr + i), args.max_records);
+        const int r0 = record_offset(args.tile_ptr, i, args.max_records);
         s_r0[t] = r0;
-        s_cnt[t] = (int)min((long long)__ldg(args.tile_ptr + i + 1), args.max_records) - r0;
+        s_cnt[t] = record_offset(args.tile_ptr, i + 1, args.max_records) - r0;
     }
     pdl_wait();  // phase A's workspace writes are complete and visible
     __syncthreads();
