@@ -3,9 +3,12 @@
 // (Sec. 3.1), from which the correspondence operator of Sec. 3.2 is built.
 //
 // A z-buffer over pixel centres, in two kernels:
-//  raster_faces_kernel: one thread per (face, view).  The face is projected;
-//    every pixel centre inside or on it (three sign-normalised edge
-//    functions) gets the camera z of the ray / face-plane intersection, and
+//  raster_faces_kernel: one thread per face, looping over the views (the
+//    face's vertices are loaded once; a CTA's faces normally belong to one
+//    asset, whose cameras are staged in shared memory).  For each view the
+//    face is projected; every pixel centre inside or on it (three
+//    sign-normalised edge functions) gets the camera z of the ray /
+//    face-plane intersection, and
 //    the key (depth bits << 32 | face index) is min-combined into the
 //    pixel's z-buffer word with a 64-bit atomicMin (nearest face wins, ties
 //    to the lower face index; positive floats order like their bits).  A
@@ -41,27 +44,28 @@ struct Cam32 {
     float R[9], t[3], fx, fy, cx, cy;
 };
 
+// c points to global or shared memory (generic loads)
 __device__ __forceinline__ Cam32 load_cam(const geocache_camera* c) {
     Cam32 k;
     const float* p = reinterpret_cast<const float*>(c);
 #pragma unroll
-    for (int i = 0; i < 9; ++i) k.R[i] = __ldg(p + i);
+    for (int i = 0; i < 9; ++i) k.R[i] = p[i];
 #pragma unroll
-    for (int i = 0; i < 3; ++i) k.t[i] = __ldg(p + 9 + i);
-    k.fx = __ldg(p + 12);
-    k.fy = __ldg(p + 13);
-    k.cx = __ldg(p + 14);
-    k.cy = __ldg(p + 15);
+    for (int i = 0; i < 3; ++i) k.t[i] = p[9 + i];
+    k.fx = p[12];
+    k.fy = p[13];
+    k.cx = p[14];
+    k.cy = p[15];
     return k;
 }
 
 // x_c = R X + t, each row summed ((R0 X0 + R1 X1) + R2 X2) + t
-__device__ __forceinline__ void cam_point(const Cam32& c, const float* X, float* xc) {
+__device__ __forceinline__ void cam_point(const Cam32& c, const float (&X)[3], float* xc) {
 #pragma unroll
     for (int r = 0; r < 3; ++r) {
-        float s = __fmul_rn(c.R[3 * r], __ldg(X));
-        s = __fadd_rn(s, __fmul_rn(c.R[3 * r + 1], __ldg(X + 1)));
-        s = __fadd_rn(s, __fmul_rn(c.R[3 * r + 2], __ldg(X + 2)));
+        float s = __fmul_rn(c.R[3 * r], X[0]);
+        s = __fadd_rn(s, __fmul_rn(c.R[3 * r + 1], X[1]));
+        s = __fadd_rn(s, __fmul_rn(c.R[3 * r + 2], X[2]));
         xc[r] = __fadd_rn(s, c.t[r]);
     }
 }
@@ -73,20 +77,13 @@ struct Face {
     int ilo, ihi, jlo, jhi;
 };
 
-// false when the face covers no pixel centre: an index outside [0, nv)
-// (reported in the status word), a vertex not in front (z <= 1e-6), zero
-// area, or a box outside the image
-__device__ __forceinline__ bool setup_face(const Cam32& c, const float* __restrict__ V, long long nv,
-                                           const int32_t* __restrict__ F, long long f, int H, int W, Face& o) {
+// false when the face covers no pixel centre: a vertex not in front
+// (z <= 1e-6), zero area, or a box outside the image
+__device__ __forceinline__ bool setup_face(const Cam32& c, const float (&X)[3][3], int H, int W, Face& o) {
     float P[3][3];
 #pragma unroll
     for (int k = 0; k < 3; ++k) {
-        const int32_t vi = __ldg(F + 3 * f + k);
-        if (vi < 0 || vi >= nv) {
-            atomicOr(&g_raster_error, 8u);
-            return false;
-        }
-        cam_point(c, V + 3 * (size_t)vi, P[k]);
+        cam_point(c, X[k], P[k]);
         if (!(P[k][2] > 1e-6f)) return false;
         o.u[k] = __fadd_rn(__fmul_rn(c.fx, __fdiv_rn(P[k][0], P[k][2])), c.cx);
         o.v[k] = __fadd_rn(__fmul_rn(c.fy, __fdiv_rn(P[k][1], P[k][2])), c.cy);
@@ -160,59 +157,83 @@ __device__ __forceinline__ int asset_of(const int64_t* __restrict__ face_off, in
     return lo;
 }
 
-__global__ void __launch_bounds__(kRasterThreads) raster_faces_kernel(
+__global__ void __launch_bounds__(kRasterThreads, 4) raster_faces_kernel(
     const float* __restrict__ V, long long nv, const int32_t* __restrict__ F, long long nf,
     const int64_t* __restrict__ face_off, int B, const geocache_camera* __restrict__ cams, int N, int H, int W,
     unsigned long long* __restrict__ zbuf) {
-    const long long f = blockIdx.x * (long long)kRasterThreads + threadIdx.x;
-    const int view = blockIdx.y;
+    __shared__ geocache_camera s_cam[GEOCACHE_MAX_VIEWS];
+    __shared__ int s_asset[2];
+    const long long f0 = blockIdx.x * (long long)kRasterThreads;
+    const long long f = f0 + threadIdx.x;
     const int lane = threadIdx.x & 31;
-    Face o;
-    Cam32 c;
-    bool live = false;
-    int b = 0;
-    if (f < nf) {
-        b = asset_of(face_off, B, f);
-        c = load_cam(cams + (size_t)b * N + view);
-        live = setup_face(c, V, nv, F, f, H, W, o);
-    }
-    const long long box = live ? (long long)(o.ihi - o.ilo + 1) * (o.jhi - o.jlo + 1) : 0;
-    unsigned long long* zb = zbuf + ((size_t)b * N + view) * (size_t)H * W;
-    if (live && box <= kSmallBox) {
-        for (int j = o.jlo; j <= o.jhi; ++j)
-            for (int i = o.ilo; i <= o.ihi; ++i) {
-                const unsigned long long key = pixel_key(c, o, i, j, (unsigned int)f);
-                if (key != kEmpty) atomicMin(zb + (size_t)j * W + i, key);
-            }
-    }
-    // large faces: the warp takes them one at a time
-    unsigned big = __ballot_sync(0xffffffffu, live && box > kSmallBox);
-    while (big) {
-        const int src = __ffs(big) - 1;
-        big &= big - 1;
-        Face q;
+    // the CTA's faces belong to one asset unless it straddles a boundary
+    if (threadIdx.x == 0) s_asset[0] = asset_of(face_off, B, f0);
+    if (threadIdx.x == 1) s_asset[1] = asset_of(face_off, B, min(f0 + kRasterThreads, nf) - 1);
+    __syncthreads();
+    const bool one_asset = s_asset[0] == s_asset[1];
+    for (int i = threadIdx.x; i < N * 16; i += kRasterThreads)
+        reinterpret_cast<float*>(s_cam)[i] = __ldg(reinterpret_cast<const float*>(cams + (size_t)s_asset[0] * N) + i);
+    __syncthreads();
+    int b = s_asset[0];
+    bool ok = f < nf;
+    float X[3][3];
+    if (ok) {
+        if (!one_asset) b = asset_of(face_off, B, f);
 #pragma unroll
         for (int k = 0; k < 3; ++k) {
-            q.u[k] = __shfl_sync(0xffffffffu, o.u[k], src);
-            q.v[k] = __shfl_sync(0xffffffffu, o.v[k], src);
-            q.n[k] = __shfl_sync(0xffffffffu, o.n[k], src);
+            const int32_t vi = __ldg(F + 3 * f + k);
+            if (vi < 0 || vi >= nv) {
+                atomicOr(&g_raster_error, 8u);
+                ok = false;
+                break;
+            }
+            X[k][0] = __ldg(V + 3 * (size_t)vi);
+            X[k][1] = __ldg(V + 3 * (size_t)vi + 1);
+            X[k][2] = __ldg(V + 3 * (size_t)vi + 2);
         }
-        q.area = __shfl_sync(0xffffffffu, o.area, src);
-        q.nd = __shfl_sync(0xffffffffu, o.nd, src);
-        q.ilo = __shfl_sync(0xffffffffu, o.ilo, src);
-        q.ihi = __shfl_sync(0xffffffffu, o.ihi, src);
-        q.jlo = __shfl_sync(0xffffffffu, o.jlo, src);
-        q.jhi = __shfl_sync(0xffffffffu, o.jhi, src);
-        const int qb = __shfl_sync(0xffffffffu, b, src);
-        const long long qf = __shfl_sync(0xffffffffu, f, src);
-        const Cam32 qc = load_cam(cams + (size_t)qb * N + view);
-        unsigned long long* qz = zbuf + ((size_t)qb * N + view) * (size_t)H * W;
-        const int bw = q.ihi - q.ilo + 1;
-        const long long n = (long long)bw * (q.jhi - q.jlo + 1);
-        for (long long k = lane; k < n; k += 32) {
-            const int i = q.ilo + (int)(k % bw), j = q.jlo + (int)(k / bw);
-            const unsigned long long key = pixel_key(qc, q, i, j, (unsigned int)qf);
-            if (key != kEmpty) atomicMin(qz + (size_t)j * W + i, key);
+    }
+    for (int view = 0; view < N; ++view) {
+        Face o;
+        const Cam32 c = load_cam(b == s_asset[0] ? s_cam + view : cams + (size_t)b * N + view);
+        const bool live = ok && setup_face(c, X, H, W, o);
+        const long long box = live ? (long long)(o.ihi - o.ilo + 1) * (o.jhi - o.jlo + 1) : 0;
+        unsigned long long* zb = zbuf + ((size_t)b * N + view) * (size_t)H * W;
+        if (live && box <= kSmallBox) {
+            for (int j = o.jlo; j <= o.jhi; ++j)
+                for (int i = o.ilo; i <= o.ihi; ++i) {
+                    const unsigned long long key = pixel_key(c, o, i, j, (unsigned int)f);
+                    if (key != kEmpty) atomicMin(zb + (size_t)j * W + i, key);
+                }
+        }
+        // large faces: the warp takes them one at a time
+        unsigned big = __ballot_sync(0xffffffffu, live && box > kSmallBox);
+        while (big) {
+            const int src = __ffs(big) - 1;
+            big &= big - 1;
+            Face q;
+#pragma unroll
+            for (int k = 0; k < 3; ++k) {
+                q.u[k] = __shfl_sync(0xffffffffu, o.u[k], src);
+                q.v[k] = __shfl_sync(0xffffffffu, o.v[k], src);
+                q.n[k] = __shfl_sync(0xffffffffu, o.n[k], src);
+            }
+            q.area = __shfl_sync(0xffffffffu, o.area, src);
+            q.nd = __shfl_sync(0xffffffffu, o.nd, src);
+            q.ilo = __shfl_sync(0xffffffffu, o.ilo, src);
+            q.ihi = __shfl_sync(0xffffffffu, o.ihi, src);
+            q.jlo = __shfl_sync(0xffffffffu, o.jlo, src);
+            q.jhi = __shfl_sync(0xffffffffu, o.jhi, src);
+            const int qb = __shfl_sync(0xffffffffu, b, src);
+            const long long qf = __shfl_sync(0xffffffffu, f, src);
+            const Cam32 qc = load_cam(qb == s_asset[0] ? s_cam + view : cams + (size_t)qb * N + view);
+            unsigned long long* qz = zbuf + ((size_t)qb * N + view) * (size_t)H * W;
+            const int bw = q.ihi - q.ilo + 1;
+            const long long n = (long long)bw * (q.jhi - q.jlo + 1);
+            for (long long k = lane; k < n; k += 32) {
+                const int i = q.ilo + (int)(k % bw), j = q.jlo + (int)(k / bw);
+                const unsigned long long key = pixel_key(qc, q, i, j, (unsigned int)qf);
+                if (key != kEmpty) atomicMin(qz + (size_t)j * W + i, key);
+            }
         }
     }
 }
@@ -271,8 +292,7 @@ cudaError_t launch_raster(const float* V, long long nv, const int32_t* F, long l
     if (nf > 0) {
         const long long gx = (nf + kRasterThreads - 1) / kRasterThreads;
         if (gx > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-        raster_faces_kernel<<<dim3((unsigned)gx, N), kRasterThreads, 0, s>>>(V, nv, F, nf, face_off, B, cams, N, H,
-                                                                              W, zbuf);
+        raster_faces_kernel<<<(unsigned)gx, kRasterThreads, 0, s>>>(V, nv, F, nf, face_off, B, cams, N, H, W, zbuf);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
