@@ -328,8 +328,13 @@ class Trajectory:
 
     def run_e2e(self, host, graph=None):
         """One trajectory from pinned host inputs to a host copy of the final
-        latents (the trajectory itself replayed from `graph` when given)."""
+        latents (the trajectory itself replayed from `graph` when given).
+        With graphs the uploads run on a copy stream in the order the steps
+        need them and each step waits only for its own inputs, so compute
+        overlaps the remaining uploads."""
         import torch
+        if graph:
+            return self._run_e2e_overlapped(host)
         self.pos.copy_(host["pos"], non_blocking=True)
         self.valid.copy_(host["valid"], non_blocking=True)
         self.cams.copy_(host["cams"], non_blocking=True)
@@ -345,6 +350,36 @@ class Trajectory:
         out = torch.empty(self.x.shape, dtype=self.x.dtype, pin_memory=True)
         out.copy_(self.x, non_blocking=True)
         torch.cuda.current_stream().synchronize()
+        return out
+
+    def _run_e2e_overlapped(self, host):
+        import torch
+        cur = torch.cuda.current_stream()
+        if getattr(self, "copy_stream", None) is None:
+            self.copy_stream = torch.cuda.Stream()
+        cs = self.copy_stream
+        cs.wait_stream(cur)  # the previous trajectory is done with these buffers
+        ready = []
+        with torch.cuda.stream(cs):
+            for name in ("pos", "valid", "cams", "x"):
+                getattr(self, name).copy_(host[name], non_blocking=True)
+            ready.append(torch.cuda.Event())
+            ready[-1].record(cs)
+            for t in range(self.w.S):
+                if t in host["full"]:
+                    self.full_x0[t].copy_(host["full"][t], non_blocking=True)
+                if t in host["anchor"]:
+                    self.anchor_x0[t].copy_(host["anchor"][t], non_blocking=True)
+                ready.append(torch.cuda.Event())
+                ready[-1].record(cs)
+        cur.wait_event(ready[0])
+        self.g_build.replay()
+        for t, g in enumerate(self.g_steps):
+            cur.wait_event(ready[t + 1])
+            g.replay()
+        out = torch.empty(self.x.shape, dtype=self.x.dtype, pin_memory=True)
+        out.copy_(self.x, non_blocking=True)
+        cur.synchronize()
         return out
 
     def h2d_bytes(self):
