@@ -347,10 +347,17 @@ class Trajectory:
             self.replay()
         else:
             self.run()
-        out = torch.empty(self.x.shape, dtype=self.x.dtype, pin_memory=True)
+        out = self._host_out()
         out.copy_(self.x, non_blocking=True)
         torch.cuda.current_stream().synchronize()
         return out
+
+    def _host_out(self):
+        """Pinned host buffer of the final latents, allocated once."""
+        import torch
+        if getattr(self, "host_out", None) is None:
+            self.host_out = torch.empty(self.x.shape, dtype=self.x.dtype, pin_memory=True)
+        return self.host_out
 
     def _run_e2e_overlapped(self, host):
         import torch
@@ -377,7 +384,7 @@ class Trajectory:
         for t, g in enumerate(self.g_steps):
             cur.wait_event(ready[t + 1])
             g.replay()
-        out = torch.empty(self.x.shape, dtype=self.x.dtype, pin_memory=True)
+        out = self._host_out()
         out.copy_(self.x, non_blocking=True)
         cur.synchronize()
         return out
