@@ -127,3 +127,44 @@ def test_permutation_out_of_range_is_reported(gc, workloads):
     assert ei.value.status == gc.EINVAL
     gc.device_status()  # cleared by the read
     np.testing.assert_array_equal(shuf._keep["records"].cpu().numpy(), g.records.cpu().numpy())
+
+
+def test_shuffle_with_value_copy_interaction(gc, workloads):
+    # Table 3's "shuf + value" cell: both ablations at once
+    w = workloads("hunyuan64")
+    g = DeviceGeometry(w, K=4, tables=False)
+    tau = oracle.tau(w.pos, w.valid, w.tol_frac)
+    idx, wt, _ = oracle.build_corr(w.pos, w.valid, w.cams, tau, K=4, with_band=False)
+    perm = synth.pair_permutation(_pair_counts(g, w), seed=23)
+    shuf = gc.permute_records(g.corr, torch.from_numpy(perm).cuda())
+    anchors = oracle.rotate_anchors(w.N, w.a, 1)
+    params = synth.recon_params(w, 6)
+    (x0_prev, x0_new, xt64), got, d_xn = _gpu_step(gc, w, g, shuf, anchors, params, "copy")
+    ref_x0, ref_xn, _ = oracle.transport_step(anchors, x0_new, x0_prev, table=oracle.shuffle_rows(idx, wt, perm),
+                                              x_t=xt64, recon=recon_kw(params, None), update="copy")
+    _check(w, got, d_xn, ref_x0, ref_xn)
+
+
+@pytest.mark.parametrize("mode", ["sparse", "mask"])
+def test_value_copy_in_place(gc, workloads, mode):
+    # x0_out == x0_prev and x_next == x_t: the anchors' rows are written after
+    # the gathers, covered targets are overwritten, the rest keep their state
+    w = workloads("solids96")
+    g = DeviceGeometry(w, K=w.K)
+    anchors = oracle.rotate_anchors(w.N, w.a, 2)
+    params = synth.recon_params(w, 3)
+    x0_prev, x0_new, xt32 = step_inputs(w, 5, anchors)
+    xt64, xt_t = latent_values(xt32, w)
+    d_x0 = torch.from_numpy(x0_prev).cuda()
+    d_new = torch.from_numpy(x0_new).cuda()
+    d_x = xt_t.cuda()
+    r = gc.make_recon(params["sampler"], a_t=params.get("a_t", 0), a_prev=params.get("a_prev", 0),
+                      sigma=params.get("sigma", 0), sigma_next=params.get("sigma_next", 0))
+    gc.transport_step(g.corr_for(mode), anchors, w.C, d_new, d_x0, d_x0, d_x, d_x, r, workspace=g.workspace(w.C),
+                      update="copy")
+    torch.cuda.synchronize()
+    gc.device_status()
+    tau = oracle.tau(w.pos, w.valid, w.tol_frac)
+    ref_x0, ref_xn, _ = oracle.transport_step(anchors, x0_new, x0_prev, K=w.K, geom=(w.pos, w.valid, w.cams, tau),
+                                              x_t=xt64, recon=recon_kw(params, None), update="copy")
+    _check(w, d_x0.cpu().numpy(), d_x, ref_x0, ref_xn)
