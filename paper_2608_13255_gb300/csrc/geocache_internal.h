@@ -65,7 +65,6 @@ cudaError_t launch_permute_records(const geocache_tap_record* src, const int32_t
                                    long long n, cudaStream_t s);
 __host__ __device__ int tiles_per_view(int H, int W);
 cudaError_t launch_transport(const TransportArgs& t, cudaStream_t s);
-int transport_launch_count(int a, int C, int in_place);
 cudaError_t launch_copy_anchor_rows(const TransportArgs& t, cudaStream_t s);
 cudaError_t launch_reconstruct(const void* x_t, const float* x0, void* x_next, int lat_dtype, int64_t n,
                                const ReconCoef& coef, float* pred_out, float* x0_store, cudaStream_t s);

@@ -1347,8 +1347,6 @@ static cudaError_t launch_transport_t(const TransportArgs& t, cudaStream_t s) {
     }
 }
 
-int transport_launch_count(int, int, int in_place) { return 1 + (in_place ? 1 : 0); }
-
 cudaError_t launch_transport(const TransportArgs& t, cudaStream_t s) {
     if (t.lat_dtype == GEOCACHE_BF16)
         return t.K == 4 ? launch_transport_t<__nv_bfloat16, 4>(t, s) : launch_transport_t<__nv_bfloat16, 1>(t, s);

@@ -448,8 +448,11 @@ def transport_launches(a: int, N: int, mode: int, in_place: bool = False) -> int
 
 
 def device_status(stream=None):
-    """geocache_device_status: raise GeocacheError(ETIMEOUT) if a kernel's
-    bounded wait gave up since the last check."""
+    """geocache_device_status (synchronises, reads and clears the device
+    status word): raises GeocacheError with ESHAPE (a sparse build overflowed
+    max_records), EINVAL (a record permutation entry or a mesh face index was
+    out of range) or ETIMEOUT (a kernel's bounded wait gave up) for what
+    happened since the last check."""
     _check(load().geocache_device_status(_stream(stream)))
 
 
