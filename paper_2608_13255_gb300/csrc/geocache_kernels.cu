@@ -80,7 +80,7 @@ __device__ __forceinline__ void box_reduce_warp(Box& x) {
 }
 
 __global__ void __launch_bounds__(512) tau_kernel(const float* __restrict__ pos, const uint8_t* __restrict__ valid,
-                                                  int N, int HW, float tol_frac, float* __restrict__ tau) {
+                                                  int N, int HW, float tol_frac, int quads, float* __restrict__ tau) {
     namespace cg = cooperative_groups;
     cg::cluster_group cluster = cg::this_cluster();
     const int cs = (int)cluster.num_blocks();
@@ -94,14 +94,36 @@ __global__ void __launch_bounds__(512) tau_kernel(const float* __restrict__ pos,
     x.any = 0;
     for (int v = rank; v < N; v += cs) {
         const size_t base = ((size_t)b * N + v) * HW;
-        for (int i = threadIdx.x; i < HW; i += blockDim.x) {
-            if (!__ldg(valid + base + i)) continue;
-            x.any = 1;
+        if (quads) {  // four texels per load: their 4 validity bytes and 12 position floats
+            const uint32_t* vq = reinterpret_cast<const uint32_t*>(valid + base);
+            const float4* pq = reinterpret_cast<const float4*>(pos + 3 * base);
+#pragma unroll 4
+            for (int i = threadIdx.x; i < HW / 4; i += blockDim.x) {
+                const uint32_t m = __ldg(vq + i);
+                if (!m) continue;
+                x.any = 1;
+                const float4 f0 = __ldg(pq + 3 * i), f1 = __ldg(pq + 3 * i + 1), f2 = __ldg(pq + 3 * i + 2);
+                const float f[12] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w, f2.x, f2.y, f2.z, f2.w};
 #pragma unroll
-            for (int c = 0; c < 3; ++c) {
-                const float p = __ldg(pos + 3 * (base + i) + c);
-                x.lo[c] = fminf(x.lo[c], p);
-                x.hi[c] = fmaxf(x.hi[c], p);
+                for (int k = 0; k < 4; ++k) {
+                    if (!((m >> (8 * k)) & 0xffu)) continue;
+#pragma unroll
+                    for (int c = 0; c < 3; ++c) {
+                        x.lo[c] = fminf(x.lo[c], f[3 * k + c]);
+                        x.hi[c] = fmaxf(x.hi[c], f[3 * k + c]);
+                    }
+                }
+            }
+        } else {
+            for (int i = threadIdx.x; i < HW; i += blockDim.x) {
+                if (!__ldg(valid + base + i)) continue;
+                x.any = 1;
+#pragma unroll
+                for (int c = 0; c < 3; ++c) {
+                    const float p = __ldg(pos + 3 * (base + i) + c);
+                    x.lo[c] = fminf(x.lo[c], p);
+                    x.hi[c] = fmaxf(x.hi[c], p);
+                }
             }
         }
     }
@@ -158,7 +180,9 @@ cudaError_t launch_tau(const float* pos, const uint8_t* valid, int B, int N, int
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, tau_kernel, pos, valid, N, H * W, tol_frac, tau);
+    // quads: every view's texels start on a 4-texel boundary with 16-byte aligned positions
+    const int quads = (H * W) % 4 == 0 && (uintptr_t)pos % 16 == 0 && (uintptr_t)valid % 4 == 0;
+    return cudaLaunchKernelEx(&cfg, tau_kernel, pos, valid, N, H * W, tol_frac, quads, tau);
 }
 
 // ------------------------------------------------------- correspondence --
@@ -256,52 +280,41 @@ __device__ __forceinline__ int tiles_per_view_dev(int H, int W) {
 // when the total does not fit an int32
 __global__ void __launch_bounds__(1024) exclusive_scan_kernel(int32_t* a, long long n) {
     __shared__ long long s_warp[32];
-    __shared__ long long s_carry;
-    constexpr int kItems = 16;
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    if (t == 0) s_carry = 0;
-    __syncthreads();
-    for (long long base = 0; base < n; base += 1024LL * kItems) {
-        int v[kItems];
-        long long sum = 0;
+    // thread t owns the contiguous segment [lo, hi): its sum, one block-wide
+    // exclusive scan of the sums, then the segment rewritten from its offset
+    const long long per = (n + 1023) / 1024;
+    const long long lo = min(n, (long long)t * per), hi = min(n, lo + per);
+    long long sum = 0;
+    for (long long i = lo; i < hi; ++i) sum += a[i];
+    long long incl = sum;
 #pragma unroll
-        for (int i = 0; i < kItems; ++i) {
-            const long long idx = base + (long long)t * kItems + i;
-            v[i] = idx < n ? a[idx] : 0;
-            sum += v[i];
-        }
-        long long incl = sum;
+    for (int off = 1; off < 32; off <<= 1) {
+        const long long y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
+    }
+    if (lane == 31) s_warp[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+        long long w = s_warp[lane];
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
-            const long long y = __shfl_up_sync(0xffffffffu, incl, off);
-            if (lane >= off) incl += y;
+            const long long y = __shfl_up_sync(0xffffffffu, w, off);
+            if (lane >= off) w += y;
         }
-        if (lane == 31) s_warp[warp] = incl;
-        __syncthreads();
-        if (warp == 0) {
-            long long w = s_warp[lane];
-#pragma unroll
-            for (int off = 1; off < 32; off <<= 1) {
-                const long long y = __shfl_up_sync(0xffffffffu, w, off);
-                if (lane >= off) w += y;
-            }
-            s_warp[lane] = w;
-        }
-        __syncthreads();
-        long long run = s_carry + (warp ? s_warp[warp - 1] : 0) + incl - sum;
-#pragma unroll
-        for (int i = 0; i < kItems; ++i) {
-            const long long idx = base + (long long)t * kItems + i;
-            if (idx < n) a[idx] = run > 0x7fffffffLL ? -1 : (int32_t)run;
-            run += v[i];
-        }
-        __syncthreads();
-        if (t == 0) s_carry += s_warp[31];
-        __syncthreads();
+        s_warp[lane] = w;
     }
-    if (t == 0) {
-        a[n] = s_carry > 0x7fffffffLL ? -1 : (int32_t)s_carry;
-        if (s_carry > 0x7fffffffLL) atomicOr(&g_device_error, 2u);  // more records than int32 offsets index
+    __syncthreads();
+    long long run = (warp ? s_warp[warp - 1] : 0) + incl - sum;
+    for (long long i = lo; i < hi; ++i) {
+        const int x = a[i];
+        a[i] = run > 0x7fffffffLL ? -1 : (int32_t)run;
+        run += x;
+    }
+    if (t == 1023) {
+        const long long total = s_warp[31];
+        a[n] = total > 0x7fffffffLL ? -1 : (int32_t)total;
+        if (total > 0x7fffffffLL) atomicOr(&g_device_error, 2u);  // more records than int32 offsets index
     }
 }
 
