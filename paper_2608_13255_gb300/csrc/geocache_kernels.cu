@@ -1137,8 +1137,18 @@ __device__ __forceinline__ void apply_records(const TransportArgs& args, int pai
 
 // Phase A: n_apply record-slice CTAs and n_stream anchor-view CTAs (tiles of
 // kTileTokens tokens), interleaved evenly in block order.
+// Resident CTAs per SM the phases are compiled for, by latent type: with
+// bf16 latents 6 (phase A, at most 40 registers) and 5 (phase B) put more
+// gathers and streamed rows in flight than the few spilled registers cost
+// (measured: unbounded, 62 / 56 registers, was 2-3 us slower per step); f32
+// latents need more registers per quad and are left unbounded.
+template <typename T>
+constexpr int kPhaseABlocks = sizeof(T) == 2 ? 6 : 1;
+template <typename T>
+constexpr int kPhaseBBlocks = sizeof(T) == 2 ? 5 : 1;
+
 template <typename T, int K, bool VEC, bool COPY>
-__global__ void __launch_bounds__(kThreads) sparse_phase_a_kernel(const TransportArgs args, int n_apply,
+__global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_kernel(const TransportArgs args, int n_apply,
                                                                   int n_stream, int n_slices) {
     pdl_launch_dependents();
     const long long total = (long long)n_apply + n_stream;
@@ -1172,7 +1182,7 @@ __global__ void __launch_bounds__(kThreads) sparse_phase_a_kernel(const Transpor
 // anchor set (fold the tile's increments); blockIdx.y >= N - a: anchor views
 // (only for an in-place cache update, see phase A).
 template <typename T, bool VEC>
-__global__ void __launch_bounds__(kThreads) sparse_phase_b_kernel(const TransportArgs args) {
+__global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_kernel(const TransportArgs args) {
     __shared__ float s_acc[kTileTokens][4];
     __shared__ uint8_t s_n[kTileTokens];
     __shared__ int s_r0[GEOCACHE_MAX_VIEWS], s_cnt[GEOCACHE_MAX_VIEWS];
@@ -1211,6 +1221,15 @@ __global__ void __launch_bounds__(kThreads) sparse_phase_b_kernel(const Transpor
     __syncthreads();
     int total = 0;
     for (int s2 = 0; s2 < a; ++s2) total += s_cnt[s2];
+    if (total == 0) {  // no record in the tile: every token keeps x0(t-1), nothing to fold
+        if (cnt > 0)
+            for (int cg = 0; cg < C; cg += 4) {
+                const int cn = C - cg < 4 ? C - cg : 4;
+                if (cg > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
+                q.store(args, b, v, p0, cnt, cg, cn);
+            }
+        return;
+    }
     for (int cg = 0; cg < C; cg += 4) {
         const int cn = C - cg < 4 ? C - cg : 4;
         if (cg > 0 && cnt > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
