@@ -100,6 +100,38 @@ def step_bytes(w):
     return non + anc
 
 
+def measure_stages(traj, reps=20):
+    """Graph-replay time of the trajectory's other stages: the correspondence
+    build (tau, keep masks and tile counts, offsets, records) and one full
+    step (the sampler reconstruction of every view from the denoiser's x0:
+    x_t and x0 read, x_{t-1} written, 4 + 2 * 2 bytes per bf16 element)."""
+    import torch
+    w = traj.w
+    full_t = next(t for t in range(w.S) if t not in traj.anchor_x0)
+    lb = 2 if w.dtype == "bf16" else 4
+    out = {}
+    for name, g, nbytes in (("build", traj.g_build, None),
+                            ("full_step", traj.g_steps[full_t], w.B * w.N * w.C * w.H * w.W * (4 + 2 * lb))):
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            g.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1) * 1e3)
+        us = statistics.median(ts)
+        out[name] = {"us": us}
+        if nbytes:
+            out[name].update({"alg_bytes": nbytes, "GBs": nbytes / us / 1e3,
+                              "frac_of_peak": nbytes / us / 1e3 / measured_peak()[0]})
+    out["what"] = "median of %d graph replays, %d assets" % (reps, w.B)
+    return out
+
+
 def measure_ablations(traj, reps=24):
     """Cached-step time of the two ablation modes of Sec. 4.3 (value copy,
     shuffled correspondence) beside the delta transport, on the bench's
@@ -644,6 +676,7 @@ def main():
         del srcs, sls
 
     ablations = measure_ablations(traj) if rank == 0 and args.corr == "sparse" else None
+    stages = measure_stages(traj) if rank == 0 and use_graphs else None
     raster = None
     if rank == 0 and not args.no_raster:
         from paper_2608_13255_gb300 import synth
@@ -683,6 +716,7 @@ def main():
                      "frac_of_8TBs": achieved / 8000.0},
         "gpu_launches": launches,
         "pack_anchors": pack,
+        "stages": stages,
         "ablations": ablations,
         "raster_posmaps": raster,
         "clocks": clocks.summary(),
