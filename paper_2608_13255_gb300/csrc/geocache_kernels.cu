@@ -1217,6 +1217,11 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
         s_r0[t] = r0;
         s_cnt[t] = record_offset(args.tile_ptr, i + 1, args.max_records) - r0;
     }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {  // the first channel group's sums, cleared before the wait
+        *reinterpret_cast<float4*>(s_acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
+        s_n[4 * t + i] = 0;
+    }
     pdl_wait();  // phase A's workspace writes are complete and visible
     __syncthreads();
     int total = 0;
@@ -1232,13 +1237,15 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
     }
     for (int cg = 0; cg < C; cg += 4) {
         const int cn = C - cg < 4 ? C - cg : 4;
-        if (cg > 0 && cnt > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
+        if (cg > 0) {
+            if (cnt > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            *reinterpret_cast<float4*>(s_acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
-            s_n[4 * t + i] = 0;
+            for (int i = 0; i < 4; ++i) {
+                *reinterpret_cast<float4*>(s_acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
+                s_n[4 * t + i] = 0;
+            }
+            __syncthreads();
         }
-        __syncthreads();
         for (int j0 = 0; j0 < total; j0 += kThreads) {
             const int j = j0 + t;
             int s_mine = -1, lp = 0;
