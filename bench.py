@@ -42,12 +42,18 @@ def parse():
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="batch128")
-    p.add_argument("--assets", type=int, default=64, help="assets per GPU (the batch128 sweep axis)")
+    p.add_argument("--assets", type=int, default=128,
+                   help="assets per GPU (the batch128 workload's sweep axis; default its largest point)")
+    p.add_argument("--sweep", default="1,8,16,32,64",
+                   help="smaller batch sizes timed on a prefix of the batch ('' to skip)")
     p.add_argument("--corr", default="sparse", choices=["sparse", "mask", "geometry", "table"])
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-raster", action="store_true", help="skip the position-map rasteriser measurement")
-    p.add_argument("--cpu-assets", type=int, default=4, help="assets in the oracle's timed sample")
+    p.add_argument("--cpu-assets", type=int, default=24,
+                   help="assets in the oracle's timed sample for cpu_baseline (one trajectory, ~10-30 s)")
+    p.add_argument("--ref-assets", type=int, default=2,
+                   help="assets per step of the reference arm (the oracle; one trajectory each, ~1 s)")
     return p.parse_args()
 
 
@@ -89,14 +95,16 @@ def describe(w):
                                               w.sampler.upper(), json.dumps(w.schedule), w.K))
 
 
-def step_bytes(w):
-    """Algorithmic HBM bytes of one cached transport step (latents only):
+def step_bytes(w, B=None):
+    """Algorithmic HBM bytes of one cached transport step (latents only) of B
+    assets (default: the workload's):
     non-anchor element: x0_prev 4 + x0 write 4 + x_t 2 + x_next 2 (bf16) = 12 B;
     anchor element: x0_new 4 + x0_prev 4 (for the increment) + cache write 4 + 4 (latents) = 16 B."""
+    B = w.B if B is None else B
     lb = 2 if w.dtype == "bf16" else 4
     hw = w.H * w.W
-    non = w.B * (w.N - w.a) * w.C * hw * (8 + 2 * lb)
-    anc = w.B * w.a * w.C * hw * (12 + 2 * lb)
+    non = B * (w.N - w.a) * w.C * hw * (8 + 2 * lb)
+    anc = B * w.a * w.C * hw * (12 + 2 * lb)
     return non + anc
 
 
@@ -175,6 +183,55 @@ def measure_ablations(traj, reps=24):
     gc.device_status()
     out["what"] = ("one cached step, %d assets, anchors %s, %d steps per graph; value_copy reads no anchor "
                    "x0(t-1); shuffled = records permuted within each (b, v, u) pair (seed 1)" % (w.B, anchors, reps))
+    return out
+
+
+def measure_sweep(traj, sizes, reps=24):
+    """Cached-step time against the number of assets per launch (the
+    workload's batch sweep): for each size the first B' assets of the bench's
+    batch get their own correspondence build and one graph of `reps` delta
+    steps ping-ponging the x0 cache (first cached anchor set).  Below about
+    25 assets a step's bytes fit in the 129 MB L2, so the fraction of the HBM
+    peak is not a DRAM figure there."""
+    import torch
+    gc, w = traj.gc, traj.w
+    t0 = next(iter(traj.anchor_x0))
+    anchors = sorted(gc.rotate_anchors(w.N, w.a, t0, w.S, traj.sched)[0])
+    peak = measured_peak()[0]
+    out = {}
+    for bs in sorted(set(sizes) | {w.B}):
+        if bs < 1 or bs > w.B:
+            continue
+        if bs == w.B:
+            corr, wsp = traj.corr, traj.workspace
+        else:
+            corr = gc.build_sparse_corr(traj.pos[:bs], traj.valid[:bs], traj.cams[:bs], K=w.K, tol_frac=w.tol_frac)
+            wsp = torch.empty(max(corr.workspace_floats(w.C), 4), dtype=torch.float32, device=traj.dev)
+        new, x, bufs = traj.anchor_x0[t0][:bs], traj.x[:bs], [b[:bs] for b in traj.bufs]
+
+        def one(i):
+            gc.transport_step(corr, anchors, w.C, new, bufs[i % 2], bufs[(i + 1) % 2], x, x, traj.recon[t0],
+                              workspace=wsp)
+        for i in range(2):
+            one(i)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for i in range(reps):
+                one(i)
+        g.replay()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        us = e0.elapsed_time(e1) * 1e3 / reps
+        nbytes = step_bytes(w, bs)
+        out[str(bs)] = {"us_per_step": us, "alg_bytes": nbytes, "frac_of_peak": nbytes / us / 1e3 / peak,
+                        "target_pixels_per_s": bs * (w.N - w.a) * w.H * w.W / us * 1e6}
+        del g, corr
+    gc.device_status()
+    out["what"] = ("one cached delta step on the first B' assets, %d steps per graph, anchors %s; keys are B'"
+                   % (reps, anchors))
     return out
 
 
@@ -554,7 +611,7 @@ def run_reference(args):
         return 0
     from paper_2608_13255_gb300 import synth
     w = workload(args)
-    ws = synth.replicate_assets(w, args.cpu_assets)
+    ws = synth.replicate_assets(w, args.ref_assets)
     for _ in range(args.warmup):
         oracle_trajectory(ws, steps=6)
     tot_pix, tot_s = 0, 0.0
@@ -566,9 +623,9 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_s / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": describe(w), "sampled_assets": args.cpu_assets},
+            "data": "synthetic", "config": {"workload": describe(w), "sampled_assets": args.ref_assets},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": "%d of %d assets per step, whole trajectories" % (args.cpu_assets, w.B)},
+                             "sample": "%d of %d assets per step, whole trajectories" % (args.ref_assets, w.B)},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
@@ -676,6 +733,9 @@ def main():
         del srcs, sls
 
     ablations = measure_ablations(traj) if rank == 0 and args.corr == "sparse" else None
+    sweep = None
+    if rank == 0 and args.corr == "sparse" and use_graphs and args.sweep:
+        sweep = measure_sweep(traj, [int(x) for x in args.sweep.split(",")])
     stages = measure_stages(traj) if rank == 0 and use_graphs else None
     raster = None
     if rank == 0 and not args.no_raster:
@@ -718,6 +778,7 @@ def main():
         "pack_anchors": pack,
         "stages": stages,
         "ablations": ablations,
+        "batch_sweep": sweep,
         "raster_posmaps": raster,
         "clocks": clocks.summary(),
         "e2e": e2e,

@@ -1,5 +1,5 @@
 """Parity at the benchmark's full size and launch configuration: the batch128
-workload at 64 assets (the bench's default point of the workload's batch
+workload at 128 assets (the bench's default: the largest point of the workload's batch
 sweep), sparse mode, bf16 latents and an f32 cache, one cached DDIM step, on
 outputs the oracle computes one by one: tau for every asset, the keep masks
 of sampled (target, source, token) rows, and x0(t) / x_{t-1} at a sample of
@@ -17,7 +17,7 @@ from gpu_helpers import DeviceGeometry, assert_bf16_close, assert_f32_close, lat
 
 pytestmark = pytest.mark.gpu
 
-B_BENCH = 64
+B_BENCH = 128
 
 
 @pytest.fixture(scope="module")
