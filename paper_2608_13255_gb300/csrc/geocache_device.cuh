@@ -90,7 +90,9 @@ __device__ __forceinline__ bool footprint(const geocache_camera& cam, float X0, 
 
 // Per-tap tests: inside the image, non-zero weight factors, foreground
 // texel, ||P_u(q) - X||^2 <= tau2.  Returns the keep mask (bit k = tap k,
-// taps ordered TL, TR, BL, BR).
+// taps ordered TL, TR, BL, BR).  A tap's position is loaded beside its
+// validity rather than after it (a background texel's position is read and
+// ignored), so the tests wait on one round of loads, not two.
 template <int K>
 __device__ __forceinline__ int tap_mask(const Footprint& f, const float* __restrict__ pos_u,
                                         const uint8_t* __restrict__ valid_u, int H, int W, float X0, float X1,
@@ -103,9 +105,9 @@ __device__ __forceinline__ int tap_mask(const Footprint& f, const float* __restr
         if (col < 0 || col >= W || row < 0 || row >= H) continue;
         if (K == 4 && (f.ax[di] == 0.0f || f.ay[dj] == 0.0f)) continue;
         const int q = row * W + col;
-        if (!__ldg(valid_u + q)) continue;
-        if (!(sqdist(pos_u + 3 * (size_t)q, X0, X1, X2) <= tau2)) continue;
-        mask |= 1 << k;
+        const int fg = __ldg(valid_u + q) != 0;
+        const int near = sqdist(pos_u + 3 * (size_t)q, X0, X1, X2) <= tau2;
+        mask |= (fg & near) << k;
     }
     return mask;
 }

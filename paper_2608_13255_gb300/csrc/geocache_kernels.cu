@@ -277,44 +277,73 @@ __device__ __forceinline__ int tiles_per_view_dev(int H, int W) {
 }
 
 // in-place exclusive prefix sum of n counts by one CTA; a[n] = total, or -1
-// when the total does not fit an int32
+// when the total does not fit an int32.  Rounds of 1024 x kScanPer
+// consecutive counts: each thread loads its kScanPer counts (16-byte loads
+// when aligned), the CTA scans the per-thread sums, and each thread rewrites
+// its counts as offsets from the running total of the earlier rounds.
+constexpr int kScanPer = 16;
+
 __global__ void __launch_bounds__(1024) exclusive_scan_kernel(int32_t* a, long long n) {
     __shared__ long long s_warp[32];
     const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-    // thread t owns the contiguous segment [lo, hi): its sum, one block-wide
-    // exclusive scan of the sums, then the segment rewritten from its offset
-    const long long per = (n + 1023) / 1024;
-    const long long lo = min(n, (long long)t * per), hi = min(n, lo + per);
-    long long sum = 0;
-    for (long long i = lo; i < hi; ++i) sum += a[i];
-    long long incl = sum;
+    const bool vec = (reinterpret_cast<uintptr_t>(a) & 15) == 0;
+    long long carry = 0;  // sum of the counts of the earlier rounds
+    for (long long c0 = 0; c0 < n; c0 += 1024LL * kScanPer) {
+        const long long lo = c0 + (long long)t * kScanPer;
+        int x[kScanPer];
+        if (vec && lo + kScanPer <= n) {
 #pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-        const long long y = __shfl_up_sync(0xffffffffu, incl, off);
-        if (lane >= off) incl += y;
-    }
-    if (lane == 31) s_warp[warp] = incl;
-    __syncthreads();
-    if (warp == 0) {
-        long long w = s_warp[lane];
+            for (int i = 0; i < kScanPer; i += 4) {
+                const int4 q = *reinterpret_cast<const int4*>(a + lo + i);
+                x[i] = q.x; x[i + 1] = q.y; x[i + 2] = q.z; x[i + 3] = q.w;
+            }
+        } else {
+#pragma unroll
+            for (int i = 0; i < kScanPer; ++i) x[i] = lo + i < n ? a[lo + i] : 0;
+        }
+        long long sum = 0;
+#pragma unroll
+        for (int i = 0; i < kScanPer; ++i) sum += x[i];
+        long long incl = sum;
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
-            const long long y = __shfl_up_sync(0xffffffffu, w, off);
-            if (lane >= off) w += y;
+            const long long y = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += y;
         }
-        s_warp[lane] = w;
+        if (lane == 31) s_warp[warp] = incl;
+        __syncthreads();
+        if (warp == 0) {
+            long long w = s_warp[lane];
+#pragma unroll
+            for (int off = 1; off < 32; off <<= 1) {
+                const long long y = __shfl_up_sync(0xffffffffu, w, off);
+                if (lane >= off) w += y;
+            }
+            s_warp[lane] = w;
+        }
+        __syncthreads();
+        long long run = carry + (warp ? s_warp[warp - 1] : 0) + incl - sum;
+#pragma unroll
+        for (int i = 0; i < kScanPer; ++i) {  // counts -> offsets
+            const int c = x[i];
+            x[i] = run > 0x7fffffffLL ? -1 : (int32_t)run;
+            run += c;
+        }
+        if (vec && lo + kScanPer <= n) {
+#pragma unroll
+            for (int i = 0; i < kScanPer; i += 4)
+                *reinterpret_cast<int4*>(a + lo + i) = make_int4(x[i], x[i + 1], x[i + 2], x[i + 3]);
+        } else {
+#pragma unroll
+            for (int i = 0; i < kScanPer; ++i)
+                if (lo + i < n) a[lo + i] = x[i];
+        }
+        carry += s_warp[31];
+        __syncthreads();  // s_warp is rewritten by the next round
     }
-    __syncthreads();
-    long long run = (warp ? s_warp[warp - 1] : 0) + incl - sum;
-    for (long long i = lo; i < hi; ++i) {
-        const int x = a[i];
-        a[i] = run > 0x7fffffffLL ? -1 : (int32_t)run;
-        run += x;
-    }
-    if (t == 1023) {
-        const long long total = s_warp[31];
-        a[n] = total > 0x7fffffffLL ? -1 : (int32_t)total;
-        if (total > 0x7fffffffLL) atomicOr(&g_device_error, 2u);  // more records than int32 offsets index
+    if (t == 0) {
+        a[n] = carry > 0x7fffffffLL ? -1 : (int32_t)carry;
+        if (carry > 0x7fffffffLL) atomicOr(&g_device_error, 2u);  // more records than int32 offsets index
     }
 }
 
@@ -328,9 +357,14 @@ cudaError_t launch_tile_ptr(const geocache_corr& c, cudaStream_t s) {
 
 // records of one (b, v, u, tile): kept rows in token order, each with its
 // footprint's top-left tap and fractions (recomputed with the same device
-// functions as the tables, so the taps and weights they give are identical)
+// functions as the tables, so the taps and weights they give are identical).
+// The tile's offsets and keep masks are loaded together, and the kept
+// targets' positions are in flight while the CTA scans its counts.  Eight
+// resident CTAs per SM (32 registers, a few spilled) hide more of that
+// latency than the unbounded 43-register build (build graph of 128 assets:
+// 620 vs 641 us).
 template <int K>
-__global__ void __launch_bounds__(256) fill_records_kernel(const float* __restrict__ pos,
+__global__ void __launch_bounds__(256, 8) fill_records_kernel(const float* __restrict__ pos,
                                                            const geocache_camera* __restrict__ cams,
                                                            const uint8_t* __restrict__ keep,
                                                            const int32_t* __restrict__ tile_ptr, int N, int H,
@@ -338,25 +372,39 @@ __global__ void __launch_bounds__(256) fill_records_kernel(const float* __restri
                                                            long long max_records) {
     const int tile = blockIdx.x, vu = blockIdx.y, b = blockIdx.z;
     const int v = vu / N, u = vu % N;
+    if (u == v) return;  // diagonal pairs have no records
     const int HW = H * W;
     const int t = threadIdx.x;
-    // the tile's first record; a tile without records (and every diagonal
-    // pair) has nothing to write
     const size_t ti = ((size_t)b * N * N + vu) * T + tile;
-    const int r_first = __ldg(tile_ptr + ti);
-    if (u == v || __ldg(tile_ptr + ti + 1) == r_first || r_first < 0) return;  // < 0: offsets overflowed (flagged)
+    const int r_first = __ldg(tile_ptr + ti), r_next = __ldg(tile_ptr + ti + 1);
+    const int p0 = tile * GEOCACHE_TILE_TOKENS + 4 * t;
+    const uint8_t* row = keep + ((size_t)b * N * N + vu) * HW;
+    uint32_t m4 = 0;  // keep masks of tokens p0 .. p0 + 3, one byte each
+    if (p0 + 3 < HW && (reinterpret_cast<uintptr_t>(row + p0) & 3) == 0) {
+        m4 = __ldg(reinterpret_cast<const uint32_t*>(row + p0));
+    } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            if (p0 + i < HW) m4 |= (uint32_t)__ldg(row + p0 + i) << (8 * i);
+    }
+    // a tile without records has nothing to write; < 0: offsets overflowed (flagged by the scan)
+    if (r_next == r_first || r_first < 0) return;
     __shared__ geocache_camera s_cam;
     __shared__ int s_warp[8];
     if (t < 16) reinterpret_cast<float*>(&s_cam)[t] = __ldg(reinterpret_cast<const float*>(cams + (size_t)b * N + u) + t);
-    const int tile0 = tile * GEOCACHE_TILE_TOKENS;
-    const uint8_t* row = keep + ((size_t)b * N * N + vu) * HW;
-    uint32_t m[4];
+    const size_t tv0 = ((size_t)b * N + v) * HW;
+    float X[4][3];
     int mine = 0;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const int p = tile0 + 4 * t + i;
-        m[i] = p < HW ? __ldg(row + p) : 0u;
-        mine += m[i] != 0;
+        X[i][0] = X[i][1] = X[i][2] = 0.0f;
+        if ((m4 >> (8 * i)) & 0xffu) {
+            const float* q = pos + 3 * (tv0 + p0 + i);
+            X[i][0] = __ldg(q);
+            X[i][1] = __ldg(q + 1);
+            X[i][2] = __ldg(q + 2);
+            ++mine;
+        }
     }
     // exclusive scan over the CTA (token order)
     const int lane = t & 31, warp = t >> 5;
@@ -371,16 +419,14 @@ __global__ void __launch_bounds__(256) fill_records_kernel(const float* __restri
     int base = 0;
     for (int w = 0; w < warp; ++w) base += s_warp[w];
     long long r = (long long)r_first + base + incl - mine;
-    const size_t tv0 = ((size_t)b * N + v) * HW;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        if (!m[i]) continue;
-        const int p = tile0 + 4 * t + i;
+        const uint32_t m = (m4 >> (8 * i)) & 0xffu;
+        if (!m) continue;
         Footprint f;
-        footprint<K>(s_cam, __ldg(pos + 3 * (tv0 + p)), __ldg(pos + 3 * (tv0 + p) + 1), __ldg(pos + 3 * (tv0 + p) + 2),
-                     H, W, f);
+        footprint<K>(s_cam, X[i][0], X[i][1], X[i][2], H, W, f);
         geocache_tap_record out;
-        out.token_mask = p | (int)(m[i] << 28);
+        out.token_mask = (p0 + i) | (int)(m << 28);
         out.q_tl = f.j0 * W + f.i0;
         out.fx = K == 4 ? f.ax[1] : 0.0f;
         out.fy = K == 4 ? f.ay[1] : 0.0f;
