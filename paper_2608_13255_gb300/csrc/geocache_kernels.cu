@@ -186,68 +186,104 @@ cudaError_t launch_tau(const float* pos, const uint8_t* valid, int B, int N, int
 }
 
 // ------------------------------------------------------- correspondence --
-// One thread per (asset b, target view v, token p), looping over the source
-// views u: the target's position is loaded once.  Writes the keep masks and
-// (when requested) the idx/w tables of every pair; with tile_cnt given, adds
-// the kept rows of each (b, v, u, tile) to its count (one atomic per warp:
-// a warp's 32 tokens lie in one tile).
+// One CTA per 256 tokens of (asset b, target view v).  The CTA's foreground
+// tokens are compacted first (warp ballots), so that thread t takes the t-th
+// foreground token and the warps that test taps are full; each such thread
+// loops over the source views u with the target's position loaded once.
+// Background tokens get empty rows from their own thread.  Writes the keep
+// masks and (when requested) the idx/w tables of every pair; with tile_cnt
+// given, adds the kept rows of each (b, v, u, tile) to its count (one atomic
+// per warp: a CTA's 256 tokens lie in one tile).
+constexpr int kBuildThreads = 256;
+static_assert(GEOCACHE_TILE_TOKENS % kBuildThreads == 0, "a build CTA's tokens lie in one tile");
+
 template <int K>
-__global__ void __launch_bounds__(256) build_corr_kernel(const float* __restrict__ pos,
+__global__ void __launch_bounds__(kBuildThreads) build_corr_kernel(const float* __restrict__ pos,
                                                          const uint8_t* __restrict__ valid,
                                                          const geocache_camera* __restrict__ cams,
                                                          const float* __restrict__ tau, int N, int H, int W,
                                                          int32_t* __restrict__ idx, float* __restrict__ wout,
                                                          uint8_t* __restrict__ keep, int32_t* __restrict__ tile_cnt) {
     const int HW = H * W;
-    const int p = blockIdx.x * blockDim.x + threadIdx.x;
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+    const int p_base = blockIdx.x * kBuildThreads;
+    const int p = p_base + t;
     const int v = blockIdx.y, b = blockIdx.z;
     __shared__ geocache_camera s_cam[GEOCACHE_MAX_VIEWS];
-    for (int i = threadIdx.x; i < N * 16; i += blockDim.x)
+    __shared__ int s_fg[kBuildThreads];
+    __shared__ int s_wcnt[kBuildThreads / 32];
+    for (int i = t; i < N * 16; i += kBuildThreads)
         reinterpret_cast<float*>(s_cam)[i] = __ldg(reinterpret_cast<const float*>(cams + (size_t)b * N) + i);
-    __syncthreads();
     const bool in = p < HW;
-    const size_t tv = ((size_t)b * N + v) * HW + (in ? p : 0);
-    const bool fg = in && __ldg(valid + tv);
+    const size_t view0 = ((size_t)b * N + v) * HW;
+    const bool fg = in && __ldg(valid + view0 + p);
+    // compaction of the foreground tokens, in token order
+    const unsigned bal = __ballot_sync(0xffffffffu, fg);
+    if (lane == 0) s_wcnt[warp] = __popc(bal);
+    __syncthreads();
+    int before = 0, n_fg = 0;
+#pragma unroll
+    for (int w = 0; w < kBuildThreads / 32; ++w) {
+        before += w < warp ? s_wcnt[w] : 0;
+        n_fg += s_wcnt[w];
+    }
+    if (fg) s_fg[before + __popc(bal & ((1u << lane) - 1u))] = t;
+    __syncthreads();
+    const bool work = t < n_fg;
+    const int pw = p_base + (work ? s_fg[t] : 0);  // this thread's foreground token
     float X0 = 0.f, X1 = 0.f, X2 = 0.f, tau2 = 0.f;
-    if (fg) {
-        X0 = __ldg(pos + 3 * tv);
-        X1 = __ldg(pos + 3 * tv + 1);
-        X2 = __ldg(pos + 3 * tv + 2);
+    if (work) {
+        X0 = __ldg(pos + 3 * (view0 + pw));
+        X1 = __ldg(pos + 3 * (view0 + pw) + 1);
+        X2 = __ldg(pos + 3 * (view0 + pw) + 2);
         const float tu = __ldg(tau + b);
         tau2 = __fmul_rn(tu, tu);
     }
     const int T = tiles_per_view(H, W);
     for (int u = 0; u < N; ++u) {
-        Taps t;
-        taps_clear(t);
+        Taps tp;
+        taps_clear(tp);
         int mask = 0;
-        if (fg && u != v) {
+        if (work && u != v) {
             const size_t su = ((size_t)b * N + u) * HW;
-            compute_taps<K>(s_cam[u], pos + 3 * su, valid + su, H, W, X0, X1, X2, tau2, t, &mask);
+            compute_taps<K>(s_cam[u], pos + 3 * su, valid + su, H, W, X0, X1, X2, tau2, tp, &mask);
         }
         if (tile_cnt) {
             const unsigned kept = __ballot_sync(0xffffffffu, mask != 0);
-            if ((threadIdx.x & 31) == 0 && kept)
-                atomicAdd(tile_cnt + (((size_t)b * N + v) * N + u) * T + (blockIdx.x * blockDim.x) / GEOCACHE_TILE_TOKENS,
-                          __popc(kept));
+            if (lane == 0 && kept)
+                atomicAdd(tile_cnt + (((size_t)b * N + v) * N + u) * T + p_base / GEOCACHE_TILE_TOKENS, __popc(kept));
         }
-        if (!in) continue;
-        const size_t row = (((size_t)b * N + v) * N + u) * HW + p;
-        if (keep) keep[row] = (uint8_t)mask;
+        const size_t row0 = (((size_t)b * N + v) * N + u) * HW;
+        if (keep) {
+            if (in && !fg) keep[row0 + p] = 0;
+            if (work) keep[row0 + pw] = (uint8_t)mask;
+        }
         if (!idx) continue;
         if (K == 4) {
-            reinterpret_cast<int4*>(idx)[row] = make_int4(t.q[0], t.q[1], t.q[2], t.q[3]);
-            reinterpret_cast<float4*>(wout)[row] = make_float4(t.w[0], t.w[1], t.w[2], t.w[3]);
+            if (in && !fg) {
+                reinterpret_cast<int4*>(idx)[row0 + p] = make_int4(-1, -1, -1, -1);
+                reinterpret_cast<float4*>(wout)[row0 + p] = make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+            if (work) {
+                reinterpret_cast<int4*>(idx)[row0 + pw] = make_int4(tp.q[0], tp.q[1], tp.q[2], tp.q[3]);
+                reinterpret_cast<float4*>(wout)[row0 + pw] = make_float4(tp.w[0], tp.w[1], tp.w[2], tp.w[3]);
+            }
         } else {
-            idx[row] = t.q[0];
-            wout[row] = t.w[0];
+            if (in && !fg) {
+                idx[row0 + p] = -1;
+                wout[row0 + p] = 0.0f;
+            }
+            if (work) {
+                idx[row0 + pw] = tp.q[0];
+                wout[row0 + pw] = tp.w[0];
+            }
         }
     }
 }
 
 cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s) {
     const int HW = c.H * c.W;
-    dim3 grid((HW + 255) / 256, c.N, c.B);
+    dim3 grid((HW + kBuildThreads - 1) / kBuildThreads, c.N, c.B);
     int32_t* cnt = nullptr;
     if (c.tile_ptr) {
         const size_t n = (size_t)c.B * c.N * c.N * tiles_per_view(c.H, c.W) + 1;
@@ -256,9 +292,11 @@ cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s) {
         cnt = c.tile_ptr;
     }
     if (c.K == 4)
-        build_corr_kernel<4><<<grid, 256, 0, s>>>(c.pos, c.valid, c.cams, c.tau, c.N, c.H, c.W, c.idx, c.w, c.keep, cnt);
+        build_corr_kernel<4><<<grid, kBuildThreads, 0, s>>>(c.pos, c.valid, c.cams, c.tau, c.N, c.H, c.W, c.idx, c.w,
+                                                            c.keep, cnt);
     else
-        build_corr_kernel<1><<<grid, 256, 0, s>>>(c.pos, c.valid, c.cams, c.tau, c.N, c.H, c.W, c.idx, c.w, c.keep, cnt);
+        build_corr_kernel<1><<<grid, kBuildThreads, 0, s>>>(c.pos, c.valid, c.cams, c.tau, c.N, c.H, c.W, c.idx, c.w,
+                                                            c.keep, cnt);
     return cudaGetLastError();
 }
 
