@@ -50,7 +50,7 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-raster", action="store_true", help="skip the position-map rasteriser measurement")
-    p.add_argument("--cpu-assets", type=int, default=24,
+    p.add_argument("--cpu-assets", type=int, default=32,
                    help="assets in the oracle's timed sample for cpu_baseline (one trajectory, ~10-30 s)")
     p.add_argument("--ref-assets", type=int, default=2,
                    help="assets per step of the reference arm (the oracle; one trajectory each, ~1 s)")
