@@ -605,6 +605,56 @@ def cpu_baseline(args, w_full):
                 args.cpu_assets, w_full.B, w_full.S, secs)}
 
 
+def _asset_subset(w, idx):
+    """Workload w restricted to the assets idx (same recipe, fewer assets)."""
+    out = type(w)(**{**w.__dict__})
+    out.B = len(idx)
+    out.cams = np.ascontiguousarray(w.cams[idx])
+    out.pos = np.ascontiguousarray(w.pos[idx])
+    out.valid = np.ascontiguousarray(w.valid[idx])
+    return out
+
+
+def _oracle_worker(w, barrier, queue):
+    """One process of the all-cores CPU baseline: the unchanged oracle over
+    its share of the assets, timed from a barrier shared by all workers."""
+    try:
+        import oracle  # noqa: F401  (loads the C core before the clock starts)
+        barrier.wait(timeout=300)
+        t0 = time.time()
+        pixels, _ = oracle_trajectory(w)
+        queue.put((pixels, t0, time.time()))
+    except Exception as exc:  # reported by the parent
+        queue.put(("error", repr(exc), 0.0))
+
+
+def cpu_baseline_all_cores(w_full, cores=None):
+    """The oracle, as it stands, on every asset of the workload with one
+    process per host core (assets are independent, so they split with no
+    communication); value = all cached target view-pixels / wall time from
+    the common start to the last worker's end.  Processes are spawned (CUDA
+    is already initialised in this one)."""
+    import multiprocessing as mp
+    cores = max(1, min(cores or os.cpu_count() or 1, w_full.B))
+    ctx = mp.get_context("spawn")
+    barrier, queue = ctx.Barrier(cores), ctx.Queue()
+    parts = np.array_split(np.arange(w_full.B), cores)
+    procs = [ctx.Process(target=_oracle_worker, args=(_asset_subset(w_full, idx), barrier, queue)) for idx in parts]
+    for p in procs:
+        p.start()
+    res = [queue.get(timeout=900) for _ in procs]
+    for p in procs:
+        p.join(timeout=60)
+    bad = [r for r in res if r[0] == "error"]
+    if bad:
+        raise RuntimeError("oracle worker failed: %s" % bad[0][1])
+    pixels = sum(r[0] for r in res)
+    wall = max(r[2] for r in res) - min(r[1] for r in res)
+    return {"value": pixels / wall, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "all %d assets, one whole %d-step trajectory, %d processes of the single-threaded C oracle "
+                      "(%.1f s wall)" % (w_full.B, w_full.S, cores, wall)}
+
+
 def run_reference(args):
     rank, world, _ = dist_env()
     if rank != 0:
@@ -785,6 +835,7 @@ def main():
     }
     if not args.no_cpu and world == 1:
         line["cpu_baseline"] = cpu_baseline(args, w)
+        line["cpu_baseline_all_cores"] = cpu_baseline_all_cores(w)
     print(json.dumps(line))
     if world > 1:
         dist.destroy_process_group()
