@@ -11,10 +11,11 @@
 //    face-plane intersection, and
 //    the key (depth bits << 32 | face index) is min-combined into the
 //    pixel's z-buffer word with a 64-bit atomicMin (nearest face wins, ties
-//    to the lower face index; positive floats order like their bits).  A
-//    face whose pixel box exceeds kSmallBox pixels is handed to its whole
-//    warp, whose 32 lanes stride over the box, so that a few large faces do
-//    not serialise on one thread.
+//    to the lower face index; positive floats order like their bits).  The
+//    pixel boxes of a warp's 32 faces are concatenated (prefix sums of the
+//    box sizes) and the 32 lanes stride over the concatenation, each lane
+//    finding its pixel's face by binary search over the prefix sums, so that
+//    the work is balanced whatever the mix of small and large faces.
 //  raster_resolve_kernel: one thread per pixel; the key's depth gives the
 //    world position of the intersection.
 // Every decision and the position are binary32 with one rounding per
@@ -37,7 +38,6 @@ namespace {
 __device__ unsigned int g_raster_error = 0;
 
 constexpr int kRasterThreads = 256;
-constexpr int kSmallBox = 64;                 // pixels a single thread rasterises
 constexpr unsigned long long kEmpty = ~0ull;  // z-buffer word of an uncovered pixel
 
 struct Cam32 {
@@ -75,6 +75,13 @@ __device__ __forceinline__ void cam_point(const Cam32& c, const float (&X)[3], f
 struct Face {
     float u[3], v[3], area, n[3], nd;
     int ilo, ihi, jlo, jhi;
+};
+
+// A face of a warp published for the warp's balanced pixel loop.
+struct FaceSlot {
+    Face o;
+    int b;           // asset
+    unsigned int f;  // face index (low 32 bits of the z-buffer key)
 };
 
 // false when the face covers no pixel centre: a vertex not in front
@@ -163,6 +170,8 @@ __global__ void __launch_bounds__(kRasterThreads, 4) raster_faces_kernel(
     unsigned long long* __restrict__ zbuf) {
     __shared__ geocache_camera s_cam[GEOCACHE_MAX_VIEWS];
     __shared__ int s_asset[2];
+    __shared__ FaceSlot s_slot[kRasterThreads];
+    __shared__ long long s_excl[kRasterThreads];
     const long long f0 = blockIdx.x * (long long)kRasterThreads;
     const long long f = f0 + threadIdx.x;
     const int lane = threadIdx.x & 31;
@@ -192,49 +201,45 @@ __global__ void __launch_bounds__(kRasterThreads, 4) raster_faces_kernel(
             X[k][2] = __ldg(V + 3 * (size_t)vi + 2);
         }
     }
+    FaceSlot* slots = s_slot + (threadIdx.x & ~31);
+    long long* excl_w = s_excl + (threadIdx.x & ~31);
     for (int view = 0; view < N; ++view) {
-        Face o;
         const Cam32 c = load_cam(b == s_asset[0] ? s_cam + view : cams + (size_t)b * N + view);
+        Face o;
         const bool live = ok && setup_face(c, X, H, W, o);
         const long long box = live ? (long long)(o.ihi - o.ilo + 1) * (o.jhi - o.jlo + 1) : 0;
-        unsigned long long* zb = zbuf + ((size_t)b * N + view) * (size_t)H * W;
-        if (live && box <= kSmallBox) {
-            for (int j = o.jlo; j <= o.jhi; ++j)
-                for (int i = o.ilo; i <= o.ihi; ++i) {
-                    const unsigned long long key = pixel_key(c, o, i, j, (unsigned int)f);
-                    if (key != kEmpty) atomicMin(zb + (size_t)j * W + i, key);
-                }
+        if (live) {
+            FaceSlot& my = s_slot[threadIdx.x];
+            my.o = o;
+            my.b = b;
+            my.f = (unsigned int)f;
         }
-        // large faces: the warp takes them one at a time
-        unsigned big = __ballot_sync(0xffffffffu, live && box > kSmallBox);
-        while (big) {
-            const int src = __ffs(big) - 1;
-            big &= big - 1;
-            Face q;
+        // prefix sums of the warp's box sizes: lane l's pixels are [excl, excl + box)
+        long long incl = box;
 #pragma unroll
-            for (int k = 0; k < 3; ++k) {
-                q.u[k] = __shfl_sync(0xffffffffu, o.u[k], src);
-                q.v[k] = __shfl_sync(0xffffffffu, o.v[k], src);
-                q.n[k] = __shfl_sync(0xffffffffu, o.n[k], src);
-            }
-            q.area = __shfl_sync(0xffffffffu, o.area, src);
-            q.nd = __shfl_sync(0xffffffffu, o.nd, src);
-            q.ilo = __shfl_sync(0xffffffffu, o.ilo, src);
-            q.ihi = __shfl_sync(0xffffffffu, o.ihi, src);
-            q.jlo = __shfl_sync(0xffffffffu, o.jlo, src);
-            q.jhi = __shfl_sync(0xffffffffu, o.jhi, src);
-            const int qb = __shfl_sync(0xffffffffu, b, src);
-            const long long qf = __shfl_sync(0xffffffffu, f, src);
-            const Cam32 qc = load_cam(qb == s_asset[0] ? s_cam + view : cams + (size_t)qb * N + view);
-            unsigned long long* qz = zbuf + ((size_t)qb * N + view) * (size_t)H * W;
-            const int bw = q.ihi - q.ilo + 1;
-            const long long n = (long long)bw * (q.jhi - q.jlo + 1);
-            for (long long k = lane; k < n; k += 32) {
-                const int i = q.ilo + (int)(k % bw), j = q.jlo + (int)(k / bw);
-                const unsigned long long key = pixel_key(qc, q, i, j, (unsigned int)qf);
-                if (key != kEmpty) atomicMin(qz + (size_t)j * W + i, key);
-            }
+        for (int off = 1; off < 32; off <<= 1) {
+            const long long y = __shfl_up_sync(0xffffffffu, incl, off);
+            if (lane >= off) incl += y;
         }
+        const long long total = __shfl_sync(0xffffffffu, incl, 31);
+        s_excl[threadIdx.x] = incl - box;
+        __syncwarp();
+        for (long long k = lane; k < total; k += 32) {
+            // the face of pixel k: the last lane whose range starts at or before k
+            // (it has a non-empty box, and k lies inside it)
+            int src = 0;
+#pragma unroll
+            for (int step = 16; step > 0; step >>= 1)
+                if (excl_w[src + step] <= k) src += step;
+            const FaceSlot& q = slots[src];
+            const int local = (int)(k - excl_w[src]);
+            const int bw = q.o.ihi - q.o.ilo + 1;
+            const int i = q.o.ilo + local % bw, j = q.o.jlo + local / bw;
+            const Cam32 qc = load_cam(q.b == s_asset[0] ? s_cam + view : cams + (size_t)q.b * N + view);
+            const unsigned long long key = pixel_key(qc, q.o, i, j, q.f);
+            if (key != kEmpty) atomicMin(zbuf + ((size_t)q.b * N + view) * (size_t)H * W + (size_t)j * W + i, key);
+        }
+        __syncwarp();  // the slots are rewritten for the next view
     }
 }
 
