@@ -35,3 +35,21 @@ def test_all_cores_oracle_baseline():
     r = bench.cpu_baseline_all_cores(w, cores=2)
     assert r["cores"] == 2 and r["kind"] == "oracle" and r["value"] > 0
     assert "all 2 assets" in r["sample"]
+
+
+def test_reference_arm_prints_one_json_line():
+    """`bench.py --impl reference` times the oracle (the reference arm) and
+    prints the contract's keys; no GPU is touched."""
+    import json
+    import subprocess
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1", "--warmup", "1",
+           "--workload", "hunyuan64", "--assets", "1", "--ref-assets", "1"]
+    res = subprocess.run(cmd, capture_output=True, text=True, timeout=600, cwd=ROOT)
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [l for l in res.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == bench.UNIT
+    assert d["value"] > 0 and d["higher_is_better"] is True and d["steps"] == 1
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
