@@ -642,7 +642,17 @@ def cpu_baseline_all_cores(w_full, cores=None):
     procs = [ctx.Process(target=_oracle_worker, args=(_asset_subset(w_full, idx), barrier, queue)) for idx in parts]
     for p in procs:
         p.start()
-    res = [queue.get(timeout=900) for _ in procs]
+    import queue as queue_mod
+    res, t_end = [], time.time() + 900
+    while len(res) < len(procs):
+        try:
+            res.append(queue.get(timeout=5))
+        except queue_mod.Empty:
+            if time.time() > t_end or not any(p.is_alive() for p in procs):
+                for p in procs:
+                    if p.is_alive():
+                        p.terminate()
+                raise RuntimeError("oracle workers ended with %d of %d results" % (len(res), len(procs)))
     for p in procs:
         p.join(timeout=60)
     bad = [r for r in res if r[0] == "error"]
