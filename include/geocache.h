@@ -373,6 +373,25 @@ int geocache_rotate_anchors(int N, int a, int step, int S, const geocache_schedu
 int geocache_device_status(void* stream);
 
 /* --------------------------------------------------------------------------
+ * geocache_debug_set_wait -- test hook of the failure handling (the paper has
+ * no counterpart; not needed in normal use).  The staged transport kernel
+ * (GEOMETRY / TABLE / MASK modes with H*W % 8 == 0 and 16-byte aligned
+ * buffers) waits for its shared-memory copies with a time limit instead of
+ * spinning forever.
+ *   limit_ns         limit of those waits for later calls (0 = the default, 2 s).
+ *   drop_first_copy  nonzero: the next call that runs the staged kernel arms
+ *                    none of the copies of its first unit (asset 0, view 0,
+ *                    first tile, first channel group), so that wait runs out
+ *                    for certain; its CTA sets the timeout bit of the device
+ *                    status word (geocache_device_status then returns
+ *                    GEOCACHE_ETIMEOUT) and returns without writing the
+ *                    outputs of its units, and the context stays usable.  The
+ *                    request is consumed by that call.
+ * Process-wide, not thread safe.  Returns GEOCACHE_OK.
+ * ------------------------------------------------------------------------ */
+int geocache_debug_set_wait(uint64_t limit_ns, int drop_first_copy);
+
+/* --------------------------------------------------------------------------
  * geocache_transport_step_noalloc -- geocache_transport_step for callers that
  * cannot supply a workspace (the paper has no counterpart; this is a service
  * of the library).  Some callers cannot obtain a device buffer where they run
@@ -383,10 +402,15 @@ int geocache_device_status(void* stream);
  * scratch is a fixed array of GEOCACHE_NOALLOC_MAX_WORKSPACE_FLOATS floats
  * (16 MiB) in the library's device image, present on every device that loads
  * the library until the process exits.
- *  - A step that needs more scratch (geocache_transport_workspace(corr, C)
- *    larger than the array) is rejected with GEOCACHE_ESHAPE.
+ *  - A step that needs more scratch (a sparse-mode step with a < N whose
+ *    geocache_transport_workspace(corr, C) exceeds the array) is rejected
+ *    with GEOCACHE_ESHAPE; steps that need none (a == N, other modes) are
+ *    always accepted.
  *  - The first call on each device looks up the array's device address with
  *    that device current; make that first call before any stream capture.
+ *    The address is kept for the life of the process, so the entry point
+ *    must not be used on a device after cudaDeviceReset (or any other
+ *    teardown of its primary context) in the same process.
  *  - Every call on a device shares the one array, which keeps the previous
  *    call's contents; nothing in it needs to start at zero (each entry a call
  *    reads is written earlier in the same call), but calls that overlap on

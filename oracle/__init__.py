@@ -65,6 +65,8 @@ def _lib():
         lib.oracle_transport_step.restype = i
         lib.oracle_raster.argtypes = [_P, i, _P, i, _P, i, i, _P, _P]
         lib.oracle_raster.restype = i
+        lib.oracle_pool.argtypes = [_P, _P, i, i, i, _P, _P]
+        lib.oracle_pool.restype = i
         lib.oracle_round_bf16.argtypes = [_P, _P, l]
         lib.oracle_round_bf16.restype = None
         _LIB = lib
@@ -237,6 +239,48 @@ def raster_views(V, F, cams, H, W):
     """raster() for each camera of cams [N,16]: ([N,H,W,3], [N,H,W])."""
     out = [raster(V, F, c, H, W) for c in np.asarray(cams).reshape(-1, 16)]
     return np.stack([o[0] for o in out]), np.stack([o[1] for o in out])
+
+
+def pool(pos_hi, valid_hi, s):
+    """Token-grid position map and validity from maps rendered at s times
+    the token resolution: pos_hi [..., H*s, W*s, 3], valid_hi [..., H*s, W*s]
+    -> ([..., H, W, 3] f32, [..., H, W] u8).  A token's position is the
+    binary32 mean of its valid pixels' positions (row-major order); it is
+    foreground when at least half of its s*s pixels are (see oracle_pool)."""
+    pos_hi = _c(pos_hi, np.float32)
+    valid_hi = _c(valid_hi, np.uint8)
+    Hs, Ws = valid_hi.shape[-2:]
+    if Hs % s or Ws % s or pos_hi.shape != valid_hi.shape + (3,):
+        raise ValueError("maps of %s are not an s=%d super-sampling" % (valid_hi.shape, s))
+    H, W = Hs // s, Ws // s
+    lead = valid_hi.shape[:-2]
+    pos = np.zeros(lead + (H, W, 3), np.float32)
+    valid = np.zeros(lead + (H, W), np.uint8)
+    ph, vh = pos_hi.reshape(-1, Hs, Ws, 3), valid_hi.reshape(-1, Hs, Ws)
+    po, vo = pos.reshape(-1, H, W, 3), valid.reshape(-1, H, W)
+    for k in range(ph.shape[0]):
+        rc = _lib().oracle_pool(ph[k].ctypes.data, vh[k].ctypes.data, H, W, int(s), po[k].ctypes.data,
+                                vo[k].ctypes.data)
+        if rc != 0:
+            raise ValueError("oracle_pool: %d" % rc)
+    return pos, valid
+
+
+def scaled_camera(cam, s):
+    """The camera of an s-times finer pixel grid: focal lengths and principal
+    point multiplied by s in binary32 (token (i, j) of the coarse grid covers
+    pixels (i s .. i s + s - 1, j s .. j s + s - 1) of the fine one)."""
+    c = np.array(cam, np.float32).reshape(-1, 16).copy()
+    c[:, 12:16] = c[:, 12:16] * np.float32(s)
+    return c.reshape(np.shape(cam))
+
+
+def raster_supersampled(V, F, cams, H, W, s):
+    """Token-grid maps of a mesh from renders at s times the token
+    resolution: raster() with scaled_camera(cam, s) at (H s, W s), then
+    pool().  cams [N,16] -> ([N,H,W,3], [N,H,W])."""
+    hi = raster_views(V, F, scaled_camera(np.asarray(cams).reshape(-1, 16), s), H * s, W * s)
+    return pool(hi[0], hi[1], s)
 
 
 def round_bf16(x) -> np.ndarray:

@@ -541,3 +541,38 @@ int oracle_raster(const float* V, int nv, const int32_t* F, int nf, const float*
     free(owner);
     return 0;
 }
+
+/* ---------------------------------------------------------------- pooling --
+ * Position maps rendered at image resolution brought to the latent token
+ * grid (Sec. 3.1: the pipeline renders its position maps at image
+ * resolution, an s-fold super-sampling of the token grid; Sec. 3.2: the
+ * correspondence operator acts on the token grid).  Token (i, j) covers the
+ * s x s image pixels (i s + sx, j s + sy), 0 <= sx, sy < s.  Its position is
+ * the mean of the positions of its valid pixels: summed componentwise in
+ * binary32, pixel rows sy ascending and within a row sx ascending, then
+ * divided once by their number n (binary32, correctly rounded).  It is
+ * foreground when at least half of its s*s pixels are valid (2 n >= s*s);
+ * background tokens get position 0.
+ * pos_hi [H*s, W*s, 3], valid_hi [H*s, W*s] -> pos [H, W, 3], valid [H, W].
+ * Returns 0, or -1 on bad arguments. */
+int oracle_pool(const float* pos_hi, const uint8_t* valid_hi, int H, int W, int s, float* pos, uint8_t* valid) {
+    if (!pos_hi || !valid_hi || !pos || !valid || H <= 0 || W <= 0 || s <= 0) return -1;
+    const size_t Ws = (size_t)W * s;
+    for (int j = 0; j < H; ++j)
+        for (int i = 0; i < W; ++i) {
+            float sum[3] = {0.0f, 0.0f, 0.0f};
+            int n = 0;
+            for (int sy = 0; sy < s; ++sy)
+                for (int sx = 0; sx < s; ++sx) {
+                    const size_t q = ((size_t)j * s + sy) * Ws + (size_t)i * s + sx;
+                    if (!valid_hi[q]) continue;
+                    for (int c = 0; c < 3; ++c) sum[c] = sum[c] + pos_hi[3 * q + c];
+                    ++n;
+                }
+            const size_t p = (size_t)j * W + i;
+            const int fg = 2 * n >= s * s && n > 0;
+            valid[p] = (uint8_t)fg;
+            for (int c = 0; c < 3; ++c) pos[3 * p + c] = fg ? sum[c] / (float)n : 0.0f;
+        }
+    return 0;
+}

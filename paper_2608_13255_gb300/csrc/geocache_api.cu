@@ -136,6 +136,11 @@ int geocache_device_status(void* stream) {
 
 const char* geocache_last_error(void) { return g_last_error.c_str(); }
 
+int geocache_debug_set_wait(uint64_t limit_ns, int drop_first_copy) {
+    geocache::set_debug_wait((unsigned long long)limit_ns, drop_first_copy);
+    return ok();
+}
+
 int geocache_build_corr(geocache_corr* c, void* stream) {
     if (!c) return fail(GEOCACHE_EINVAL, "corr is NULL");
     int st = check_sizes(c->B, c->N, c->H, c->W);

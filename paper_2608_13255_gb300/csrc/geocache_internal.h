@@ -26,6 +26,8 @@ struct TransportArgs {
     int write_anchor_rows;              // 0 when x0_out aliases x0_prev (rows written afterwards)
     int lat_dtype;                      // geocache_dtype
     int update;                         // geocache_update (Eq. 1 or the value-copy ablation)
+    int drop_first_copy;                // test hook: unit 0's staged copies are not issued
+    unsigned long long wait_limit_ns;   // limit of the bounded waits
     const float* pos;
     const uint8_t* valid;
     const geocache_camera* cams;
@@ -70,6 +72,8 @@ cudaError_t launch_reconstruct(const void* x_t, const float* x0, void* x_next, i
                                const ReconCoef& coef, float* pred_out, float* x0_store, cudaStream_t s);
 
 cudaError_t read_device_error(unsigned int* out, bool clear, cudaStream_t s);
+// test hook of the bounded waits (geocache_debug_set_wait)
+void set_debug_wait(unsigned long long limit_ns, int drop_first_copy);
 cudaError_t read_raster_error(unsigned int* out, bool clear, cudaStream_t s);
 cudaError_t launch_raster(const float* V, long long nv, const int32_t* F, long long nf, const int64_t* face_off,
                           int B, const geocache_camera* cams, int N, int H, int W, unsigned long long* zbuf,

@@ -6,6 +6,7 @@
 
 #include <cooperative_groups.h>
 
+#include <atomic>
 #include <cfloat>
 #include <cstdint>
 
@@ -639,7 +640,18 @@ static_assert(kTileTokens == GEOCACHE_TILE_TOKENS, "tile of the sparse form");
 constexpr int kChunk = 4;                        // anchors per work-list round
 constexpr int kPairCap = kChunk * kTileTokens;   // (token, anchor) work items of one round
 constexpr int kStages = 2;
-constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // bounded mbarrier wait: 2 s
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // default limit of a bounded mbarrier wait: 2 s
+
+// Test hook of the failure handling (geocache_debug_set_wait): the limit of
+// the bounded waits, and a one-shot request that the next staged transport
+// launch arm none of its first unit's copies, so that wait runs out.
+static std::atomic<unsigned long long> g_wait_limit_ns{kWaitLimitNs};
+static std::atomic<int> g_drop_first_copy{0};
+
+void set_debug_wait(unsigned long long limit_ns, int drop_first_copy) {
+    g_wait_limit_ns.store(limit_ns ? limit_ns : kWaitLimitNs);
+    g_drop_first_copy.store(drop_first_copy ? 1 : 0);
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
@@ -670,12 +682,12 @@ __device__ __forceinline__ unsigned long long globaltimer() {
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
     return t;
 }
-// Wait for the phase with the given parity; false after kWaitLimitNs.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity) {
+// Wait for the phase with the given parity; false after limit_ns.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, unsigned long long limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = globaltimer();
     while (!mbar_try_wait(bar, parity))
-        if (globaltimer() - t0 > kWaitLimitNs) return false;
+        if (globaltimer() - t0 > limit_ns) return false;
     return true;
 }
 
@@ -906,6 +918,7 @@ __global__ void __launch_bounds__(kThreads) transport_fused_kernel(const Transpo
 
     // issue the bulk copies of unit u into stage st (thread 0)
     auto issue = [&](long long u, int st) {
+        if (args.drop_first_copy && u == 0) return;  // test hook: this unit's wait runs out
         const UnitCoord c = unit_coord(u, n_tiles, n_cg, N);
         const int tile0 = c.tile * kTileTokens;
         const int tile_n = HW - tile0 < kTileTokens ? HW - tile0 : kTileTokens;
@@ -947,10 +960,11 @@ __global__ void __launch_bounds__(kThreads) transport_fused_kernel(const Transpo
         const int slot = args.slot_of[c.v];
         if (slot < 0) tile_increments<K, MODE, true>(args, sh, c.b, c.v, tile0, c.cg, cn);
 
-        const bool ok = mbar_wait_bounded(&sh.bar[st], parity[st]);
+        const bool ok = mbar_wait_bounded(&sh.bar[st], parity[st], args.wait_limit_ns);
         if (__syncthreads_or(!ok)) {  // the whole CTA gives up together
             if (t == 0) atomicOr(&g_device_error, 1u);
-            for (int s2 = 0; s2 < kStages; ++s2) mbar_wait_bounded(&sh.bar[s2], parity[s2]);  // copies in flight
+            for (int s2 = 0; s2 < kStages; ++s2)  // copies in flight
+                mbar_wait_bounded(&sh.bar[s2], parity[s2], args.wait_limit_ns);
             return;
         }
         parity[st] ^= 1u;
@@ -1453,6 +1467,9 @@ static cudaError_t launch_quad(const TransportArgs& t, cudaStream_t s) {
     const long long n_units = (long long)t.B * t.N * n_tiles * n_cg;
     // TMA bulk rows need 16-byte aligned starts and sizes: HW % 8 == 0 covers bf16 rows
     if (vec && HW % 8 == 0) {
+        TransportArgs ta = t;
+        ta.wait_limit_ns = g_wait_limit_ns.load();
+        ta.drop_first_copy = g_drop_first_copy.exchange(0);
         const size_t dyn = kStages * 4 * kTileTokens * (sizeof(float) + sizeof(T));
         auto kern = transport_fused_kernel<T, K, MODE>;
         static int grid = 0;  // per instantiation and process (one device per process)
@@ -1463,7 +1480,7 @@ static cudaError_t launch_quad(const TransportArgs& t, cudaStream_t s) {
             if (!grid) return cudaErrorInvalidConfiguration;
         }
         const long long g = n_units < grid ? n_units : grid;
-        kern<<<(unsigned)g, kThreads, dyn, s>>>(t, n_tiles, n_cg, n_units);
+        kern<<<(unsigned)g, kThreads, dyn, s>>>(ta, n_tiles, n_cg, n_units);
         return cudaGetLastError();
     }
     if (n_units > 0x7fffffffLL) return cudaErrorInvalidConfiguration;

@@ -51,7 +51,8 @@ extern "C" int geocache_transport_step_noalloc(const geocache_corr* corr, const 
                                                const float* x0_anchor_new, const float* x0_prev, float* x0_out,
                                                const void* x_t, void* x_next, geocache_dtype lat_dtype,
                                                const geocache_recon* recon, void* stream) {
-    const int64_t need = geocache_transport_workspace(corr, C);
+    // only a sparse-mode step with a view outside the anchor set uses scratch
+    const int64_t need = (corr && a < corr->N) ? geocache_transport_workspace(corr, C) : 0;
     if (need > kNoallocFloats)
         return geocache::set_error(GEOCACHE_ESHAPE,
                                    "geocache_transport_step_noalloc: this step needs %lld floats of scratch but the "

@@ -70,7 +70,7 @@ EXPORTS = ("geocache_build_corr", "geocache_transport_step", "geocache_reconstru
            "geocache_rotate_anchors", "geocache_device_status", "geocache_corr_record_count",
            "geocache_transport_workspace", "geocache_transport_step_noalloc", "geocache_pack_anchors",
            "geocache_unpack_anchors", "geocache_transport_step_update", "geocache_permute_records",
-           "geocache_raster_posmaps",
+           "geocache_raster_posmaps", "geocache_debug_set_wait",
            "geocache_last_error", "geocache_abi_version")
 
 
@@ -112,6 +112,8 @@ def load():
         L.geocache_is_full_step.argtypes = [i, i, ctypes.POINTER(Schedule)]
         L.geocache_rotate_anchors.argtypes = [i, i, i, i, ctypes.POINTER(Schedule), P, ctypes.POINTER(i)]
         L.geocache_device_status.argtypes = [P]
+        L.geocache_debug_set_wait.argtypes = [ctypes.c_uint64, i]
+        L.geocache_debug_set_wait.restype = ctypes.c_int
         L.geocache_last_error.restype = ctypes.c_char_p
         L.geocache_last_error.argtypes = []
         L.geocache_abi_version.argtypes = []
@@ -454,6 +456,13 @@ def device_status(stream=None):
     out of range) or ETIMEOUT (a kernel's bounded wait gave up) for what
     happened since the last check."""
     _check(load().geocache_device_status(_stream(stream)))
+
+
+def debug_set_wait(limit_ns: int = 0, drop_first_copy: bool = False):
+    """geocache_debug_set_wait (test hook): limit of the kernels' bounded waits
+    (0 = default), and whether the next staged transport call leaves its first
+    unit's copies unissued so that its wait runs out."""
+    _check(load().geocache_debug_set_wait(int(limit_ns), 1 if drop_first_copy else 0))
 
 
 def abi_version() -> int:

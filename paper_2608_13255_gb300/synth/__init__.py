@@ -198,6 +198,43 @@ def look_at_camera(az_deg: float, el_deg: float, H: int, W: int,
     return rec.astype(np.float32)
 
 
+def camera_aligned_plane(H: int, W: int, focal: float = 64.0, depth: float = 4.0, radius_frac: float = 0.4):
+    """A fronto-parallel plane whose position map projects exactly onto the
+    token centres: camera R = I, t = (0, 0, depth / 2), focal length `focal`
+    (a power of two), principal point (W/2, H/2); token (i, j) holds the point
+    of its centre ray at camera depth `depth`, ((i + 0.5 - W/2) depth / focal,
+    (j + 0.5 - H/2) depth / focal, depth / 2).  Every coordinate and every step
+    of its projection is exact in binary32, so the projection is exactly
+    (i + 0.5, j + 0.5).  Foreground: tokens whose centre lies within
+    radius_frac * min(H, W) of the image centre.
+    Returns (cam [16] f32, pos [H, W, 3] f32, valid [H, W] u8)."""
+    cam = np.zeros(CAM_FLOATS, np.float32)
+    cam[[0, 4, 8]] = 1.0
+    cam[11] = depth / 2.0
+    cam[12:16] = (focal, focal, W / 2.0, H / 2.0)
+    jj, ii = np.meshgrid(np.arange(H, dtype=np.float64), np.arange(W, dtype=np.float64), indexing="ij")
+    du, dv = ii + 0.5 - W / 2.0, jj + 0.5 - H / 2.0
+    pos = np.stack([du * depth / focal, dv * depth / focal, np.full_like(du, depth / 2.0)], -1).astype(np.float32)
+    valid = (du * du + dv * dv <= (radius_frac * min(H, W)) ** 2).astype(np.uint8)
+    pos[valid == 0] = 0.0
+    return cam, pos, valid
+
+
+def identity_camera_pair(w: "Workload", view: int = 0, plane: bool = False) -> "Workload":
+    """A two-view workload whose views share one camera and one position map:
+    view `view` of asset 0 of w (plane=False) or camera_aligned_plane (plane=True)."""
+    if plane:
+        cam, pos, valid = camera_aligned_plane(w.H, w.W)
+    else:
+        cam, pos, valid = w.cams[0, view], w.pos[0, view], w.valid[0, view]
+    out = Workload(**{**w.__dict__})
+    out.B, out.N, out.a = 1, 2, 1
+    out.cams = np.ascontiguousarray(np.stack([cam, cam])[None], dtype=np.float32)
+    out.pos = np.ascontiguousarray(np.stack([pos, pos])[None], dtype=np.float32)
+    out.valid = np.ascontiguousarray(np.stack([valid, valid])[None], dtype=np.uint8)
+    return out
+
+
 def camera_centre(cam: np.ndarray) -> np.ndarray:
     R = cam[:9].astype(np.float64).reshape(3, 3)
     return -R.T @ cam[9:12].astype(np.float64)

@@ -403,3 +403,52 @@ def test_graph_replay_matches_eager(gc, workloads):
     torch.cuda.synchronize()
     assert torch.equal(out_g, out_e)
     assert torch.equal(xn_g.view(torch.int16), xn_e.view(torch.int16))
+
+
+@pytest.mark.parametrize("K", [4, 1])
+@pytest.mark.parametrize("scene", ["plane", "asset"])
+def test_identity_camera_reproduces_anchor_delta(gc, workloads, scene, K):
+    """Target camera equal to the anchor camera (Sec. 3.2, correspondence
+    operator): the taps sit on the target's own token, where floor(u - 0.5)
+    and the zero-weight rule decide the tap set.  'plane': positions that
+    project exactly onto the token centres (one tap, weight 1, for K = 4 as
+    for K = 1); 'asset': a rendered view duplicated (projections within
+    rounding of the centres).  Tables bit-exact against the oracle; x0^1(t) -
+    x0^1(t-1) = delta^0 at every foreground token, bit for bit where the
+    single tap has weight 1 and within 1e-5 otherwise; SPARSE, TABLE and MASK
+    modes bitwise equal."""
+    w = synth.identity_camera_pair(workloads("hunyuan64"), view=1, plane=(scene == "plane"))
+    g = DeviceGeometry(w, K=K)
+    torch.cuda.synchronize()
+    nband, _ = _compare_tables(w, g, K)
+    assert nband == 0
+    fg = w.valid[0, 1].reshape(-1) > 0
+    p = np.flatnonzero(fg)
+    idx = g.idx.cpu().numpy()[0, 1, 0].reshape(-1, K)
+    wt = g.wt.cpu().numpy()[0, 1, 0].reshape(-1, K)
+    dominant = np.take_along_axis(idx[fg], wt[fg].argmax(1)[:, None], 1)[:, 0]
+    np.testing.assert_array_equal(dominant, p)  # the heaviest tap is the target's own token
+    exact = scene == "plane" or K == 1
+    if exact:
+        np.testing.assert_array_equal(idx[fg, 0], p)
+        assert (wt[fg, 0] == 1.0).all() and (idx[fg, 1:] == -1).all()
+    else:
+        assert wt[fg].max(1).min() >= 1.0 - 1e-4
+    anchors = [0]
+    params = synth.recon_params(w, 9)
+    outs = {}
+    for mode in ("sparse", "table", "mask"):
+        _, _, got, ref = _run_step(gc, w, g, anchors, params, mode=mode)
+        outs[mode] = got
+    np.testing.assert_array_equal(outs["sparse"], outs["table"])
+    np.testing.assert_array_equal(outs["sparse"], outs["mask"])
+    x0_prev, x0_new, _ = step_inputs(w, 3, anchors)
+    got = outs["sparse"][0, 1].reshape(w.C, -1)
+    prev = x0_prev[0, 1].reshape(w.C, -1)
+    d0 = (x0_new[0, 0] - x0_prev[0, 0]).reshape(w.C, -1)  # binary32, as the kernel forms it
+    np.testing.assert_array_equal(got[:, ~fg], prev[:, ~fg])  # background keeps its state
+    if exact:  # one tap of weight 1: x0(t) = x0(t-1) + delta in binary32, bit for bit
+        np.testing.assert_array_equal(got[:, fg], (prev + d0)[:, fg])
+    err = np.abs((got.astype(np.float64) - prev)[:, fg] - d0[:, fg].astype(np.float64))
+    assert err.max() <= 1e-5, err.max()
+    print("%s K=%d: %d foreground tokens, max |x0(t) - x0(t-1) - delta| %.3g" % (scene, K, fg.sum(), err.max()))

@@ -84,6 +84,39 @@ def test_identity_camera_reproduces_anchor_delta():
         np.testing.assert_array_equal(x0_out[0, 1][:, ~fg], x0_prev[0, 1][:, ~fg])
 
 
+def test_exact_centre_projections_keep_one_tap_and_reproduce_the_delta():
+    # a camera-aligned plane whose positions project exactly onto the token
+    # centres, seen by two identical cameras: every footprint fraction is
+    # exactly 0, so the zero-weight rule leaves the single tap at the target's
+    # own token with weight 1 (K = 4 and K = 1 alike), and the target's x0
+    # changes by exactly the anchor's delta (Sec. 3.2, correspondence operator
+    # and Eq. 1 with one covering anchor)
+    w = synth.identity_camera_pair(synth.make_workload("hunyuan64", H=32, W=32), plane=True)
+    tau = oracle.tau(w.pos, w.valid)
+    fg = w.valid[0, 1].reshape(-1) > 0
+    p = np.flatnonzero(fg)
+    # the closed form of the projection: token (i, j) lands on (i + 0.5, j + 0.5)
+    cam = w.cams[0, 0]
+    for q in p[:: max(1, len(p) // 50)]:
+        uu, vv = oracle.project(cam, w.pos[0, 0].reshape(-1, 3)[q])[:2]
+        assert (uu, vv) == (q % w.W + 0.5, q // w.W + 0.5)
+    anchors = [0]
+    x0_prev, x0_new = _setup(w, anchors, seed=5)
+    d0 = x0_new[0, 0] - x0_prev[0, 0]
+    for K in (4, 1):
+        idx, wt, band = oracle.build_corr(w.pos, w.valid, w.cams, tau, K=K)
+        assert band.sum() == 0
+        row, wrow = idx[0, 1, 0].reshape(-1, K), wt[0, 1, 0].reshape(-1, K)
+        np.testing.assert_array_equal(row[fg, 0], p)
+        assert (wrow[fg, 0] == 1.0).all()
+        assert (row[fg, 1:] == -1).all() and (wrow[fg, 1:] == 0.0).all()
+        assert (row[~fg] == -1).all()
+        x0_out, _, _ = oracle.transport_step(anchors, x0_new, x0_prev, K=K, geom=(w.pos, w.valid, w.cams, tau))
+        got = (x0_out[0, 1] - x0_prev[0, 1]).reshape(w.C, -1)
+        np.testing.assert_allclose(got[:, fg], d0.reshape(w.C, -1)[:, fg], atol=1e-12, rtol=0)
+        np.testing.assert_array_equal(got[:, ~fg], 0.0)
+
+
 def test_zero_delta_leaves_targets_unchanged(workloads):
     w = workloads("hunyuan64")
     anchors = [0, 3]
