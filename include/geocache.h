@@ -303,6 +303,43 @@ int geocache_raster_posmaps(const float* verts, int64_t n_verts, const int32_t* 
                             uint64_t* zbuf, float* pos, uint8_t* valid, void* stream);
 
 /* --------------------------------------------------------------------------
+ * geocache_raster_posmaps_supersampled -- geocache_raster_posmaps rendered at
+ * s times the token grid and pooled to it.  A pipeline renders its position
+ * maps at image resolution (Sec. 3.1; e.g. 512 x 512 views for 64 x 64
+ * latents, s = 8), while the correspondence operator acts on the latent
+ * token grid (Sec. 3.2).  The faces are rasterised at (s H) x (s W) with each
+ * camera's fx, fy, cx, cy multiplied by s (binary32), under the rules of
+ * geocache_raster_posmaps; token (i, j) then covers pixels (i s + sx,
+ * j s + sy), 0 <= sx, sy < s.  Its position is the mean of the positions of
+ * its valid pixels (summed componentwise in binary32, rows sy ascending and
+ * sx ascending within a row, then divided once by their number n) and it is
+ * foreground when 2 n >= s * s; background tokens get position 0.  s = 1 is
+ * geocache_raster_posmaps.
+ *   cams      device [B, N] cameras of the token grid (H x W).
+ *   zbuf      device [B, N, s H, s W] u64 scratch (overwritten).
+ *   pos, valid  device [B, N, H, W, 3] f32 / [B, N, H, W] u8 token-grid maps.
+ * Sizes: as geocache_raster_posmaps, 1 <= s <= 16, s H and s W <= 16384.
+ * Asynchronous.  Returns GEOCACHE_OK, EINVAL, ESHAPE, EALIAS, ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_raster_posmaps_supersampled(const float* verts, int64_t n_verts, const int32_t* faces, int64_t n_faces,
+                                         const int64_t* face_off, int B, const geocache_camera* cams, int N, int H,
+                                         int W, int s, uint64_t* zbuf, float* pos, uint8_t* valid, void* stream);
+
+/* --------------------------------------------------------------------------
+ * geocache_pool_posmaps -- token-grid position maps from maps the caller
+ * rendered at s times the token resolution (Sec. 3.1 / 3.2, as above; the
+ * pooling rule of geocache_raster_posmaps_supersampled).
+ *   pos_hi, valid_hi  device [n_maps, s H, s W, 3] f32 / [n_maps, s H, s W] u8
+ *                     (valid nonzero = foreground).
+ *   pos, valid        device [n_maps, H, W, 3] f32 / [n_maps, H, W] u8.
+ * Outputs must not overlap the inputs.  Sizes: n_maps >= 0, 1 <= H, W,
+ * 1 <= s <= 16, s H and s W <= 16384.  Asynchronous.  Returns GEOCACHE_OK,
+ * EINVAL, ESHAPE, EALIAS, ECUDA.
+ * ------------------------------------------------------------------------ */
+int geocache_pool_posmaps(const float* pos_hi, const uint8_t* valid_hi, int64_t n_maps, int H, int W, int s, float* pos,
+                          uint8_t* valid, void* stream);
+
+/* --------------------------------------------------------------------------
  * geocache_reconstruct -- full-step passthrough (Sec. 3.2: at a full step the
  * denoiser runs on all N views and its x0 is both the new reference and the
  * input of the sampler conversion).

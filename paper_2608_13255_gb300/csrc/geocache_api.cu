@@ -332,31 +332,65 @@ int geocache_permute_records(const geocache_corr* c, const int32_t* perm, geocac
     return ok();
 }
 
-int geocache_raster_posmaps(const float* verts, int64_t n_verts, const int32_t* faces, int64_t n_faces,
-                            const int64_t* face_off, int B, const geocache_camera* cams, int N, int H, int W,
-                            uint64_t* zbuf, float* pos, uint8_t* valid, void* stream) {
+static int raster_entry(const char* fn, const float* verts, int64_t n_verts, const int32_t* faces, int64_t n_faces,
+                        const int64_t* face_off, int B, const geocache_camera* cams, int N, int H, int W, int ss,
+                        uint64_t* zbuf, float* pos, uint8_t* valid, void* stream) {
     if (B < 1 || B > 65535 || N < 1 || N > GEOCACHE_MAX_VIEWS || H < 1 || W < 1 || H > 16384 || W > 16384)
-        return fail(GEOCACHE_ESHAPE, "B=%d, N=%d, H=%d, W=%d out of range", B, N, H, W);
+        return fail(GEOCACHE_ESHAPE, "%s: B=%d, N=%d, H=%d, W=%d out of range", fn, B, N, H, W);
+    if (ss < 1 || ss > 16 || (int64_t)H * ss > 16384 || (int64_t)W * ss > 16384)
+        return fail(GEOCACHE_ESHAPE, "%s: s=%d out of range (1 <= s <= 16, s*H and s*W <= 16384)", fn, ss);
     if (n_verts < 0 || n_faces < 0 || n_faces > 0xffffffffLL || n_verts > 0x7fffffffLL)
-        return fail(GEOCACHE_ESHAPE, "n_verts=%lld, n_faces=%lld out of range", (long long)n_verts, (long long)n_faces);
+        return fail(GEOCACHE_ESHAPE, "%s: n_verts=%lld, n_faces=%lld out of range", fn, (long long)n_verts,
+                    (long long)n_faces);
     if (!cams || !face_off || !zbuf || !pos || !valid || (n_faces > 0 && (!verts || !faces)))
-        return fail(GEOCACHE_EINVAL, "verts, faces, face_off, cams, zbuf, pos and valid are required");
-    if ((uintptr_t)zbuf & 7) return fail(GEOCACHE_EINVAL, "zbuf must be 8-byte aligned");
+        return fail(GEOCACHE_EINVAL, "%s: verts, faces, face_off, cams, zbuf, pos and valid are required", fn);
+    if ((uintptr_t)zbuf & 7) return fail(GEOCACHE_EINVAL, "%s: zbuf must be 8-byte aligned", fn);
     const size_t px = (size_t)B * N * H * W;
     const void* outs[3] = {zbuf, pos, valid};
-    const size_t ob[3] = {px * 8, px * 12, px};
+    const size_t ob[3] = {px * ss * ss * 8, px * 12, px};
     const void* ins[5] = {verts, faces, face_off, cams, nullptr};
     const size_t ib[5] = {(size_t)n_verts * 12, (size_t)n_faces * 12, (size_t)(B + 1) * 8, sizeof(geocache_camera) * B * N, 0};
     for (int i = 0; i < 3; ++i) {
         for (int j = i + 1; j < 3; ++j)
-            if (overlap(outs[i], ob[i], outs[j], ob[j])) return fail(GEOCACHE_EALIAS, "zbuf, pos and valid overlap");
+            if (overlap(outs[i], ob[i], outs[j], ob[j])) return fail(GEOCACHE_EALIAS, "%s: zbuf, pos and valid overlap", fn);
         for (int j = 0; j < 4; ++j)
-            if (overlap(outs[i], ob[i], ins[j], ib[j])) return fail(GEOCACHE_EALIAS, "an output overlaps an input");
+            if (overlap(outs[i], ob[i], ins[j], ib[j])) return fail(GEOCACHE_EALIAS, "%s: an output overlaps an input", fn);
     }
-    cudaError_t e = geocache::launch_raster(verts, n_verts, faces, n_faces, face_off, B, cams, N, H, W,
+    cudaError_t e = geocache::launch_raster(verts, n_verts, faces, n_faces, face_off, B, cams, N, H, W, ss,
                                             reinterpret_cast<unsigned long long*>(zbuf), pos, valid,
                                             (cudaStream_t)stream);
-    if (e != cudaSuccess) return cuda_fail(e, "rasteriser launch");
+    if (e != cudaSuccess) return cuda_fail(e, fn);
+    return ok();
+}
+
+int geocache_raster_posmaps(const float* verts, int64_t n_verts, const int32_t* faces, int64_t n_faces,
+                            const int64_t* face_off, int B, const geocache_camera* cams, int N, int H, int W,
+                            uint64_t* zbuf, float* pos, uint8_t* valid, void* stream) {
+    return raster_entry("geocache_raster_posmaps", verts, n_verts, faces, n_faces, face_off, B, cams, N, H, W, 1, zbuf,
+                        pos, valid, stream);
+}
+
+int geocache_raster_posmaps_supersampled(const float* verts, int64_t n_verts, const int32_t* faces, int64_t n_faces,
+                                         const int64_t* face_off, int B, const geocache_camera* cams, int N, int H,
+                                         int W, int s, uint64_t* zbuf, float* pos, uint8_t* valid, void* stream) {
+    return raster_entry("geocache_raster_posmaps_supersampled", verts, n_verts, faces, n_faces, face_off, B, cams, N,
+                        H, W, s, zbuf, pos, valid, stream);
+}
+
+int geocache_pool_posmaps(const float* pos_hi, const uint8_t* valid_hi, int64_t n_maps, int H, int W, int s, float* pos,
+                          uint8_t* valid, void* stream) {
+    if (n_maps < 0 || H < 1 || W < 1 || H > 16384 || W > 16384)
+        return fail(GEOCACHE_ESHAPE, "geocache_pool_posmaps: n_maps=%lld, H=%d, W=%d out of range", (long long)n_maps, H, W);
+    if (s < 1 || s > 16 || (int64_t)H * s > 16384 || (int64_t)W * s > 16384)
+        return fail(GEOCACHE_ESHAPE, "geocache_pool_posmaps: s=%d out of range (1 <= s <= 16, s*H and s*W <= 16384)", s);
+    if (n_maps > 0 && (!pos_hi || !valid_hi || !pos || !valid))
+        return fail(GEOCACHE_EINVAL, "geocache_pool_posmaps: pos_hi, valid_hi, pos and valid are required");
+    const size_t tok = (size_t)n_maps * H * W, fine = tok * s * s;
+    if (overlap(pos, tok * 12, pos_hi, fine * 12) || overlap(pos, tok * 12, valid_hi, fine) ||
+        overlap(valid, tok, pos_hi, fine * 12) || overlap(valid, tok, valid_hi, fine) || overlap(pos, tok * 12, valid, tok))
+        return fail(GEOCACHE_EALIAS, "geocache_pool_posmaps: an output overlaps an input or the other output");
+    cudaError_t e = geocache::launch_pool_posmaps(pos_hi, valid_hi, n_maps, H, W, s, pos, valid, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "geocache_pool_posmaps");
     return ok();
 }
 

@@ -75,9 +75,13 @@ cudaError_t read_device_error(unsigned int* out, bool clear, cudaStream_t s);
 // test hook of the bounded waits (geocache_debug_set_wait)
 void set_debug_wait(unsigned long long limit_ns, int drop_first_copy);
 cudaError_t read_raster_error(unsigned int* out, bool clear, cudaStream_t s);
+// position maps at the token grid H x W; ss > 1: rendered at ss x H by
+// ss x W (zbuf holds B*N*H*W*ss*ss words) and pooled to the token grid
 cudaError_t launch_raster(const float* V, long long nv, const int32_t* F, long long nf, const int64_t* face_off,
-                          int B, const geocache_camera* cams, int N, int H, int W, unsigned long long* zbuf,
+                          int B, const geocache_camera* cams, int N, int H, int W, int ss, unsigned long long* zbuf,
                           float* pos, uint8_t* valid, cudaStream_t s);
+cudaError_t launch_pool_posmaps(const float* pos_hi, const uint8_t* valid_hi, long long n_maps, int H, int W, int ss,
+                                float* pos, uint8_t* valid, cudaStream_t s);
 
 // Records a status and its message for geocache_last_error(); returns status.
 int set_error(int status, const char* fmt, ...);

@@ -18,6 +18,12 @@
 //    the work is balanced whatever the mix of small and large faces.
 //  raster_resolve_kernel: one thread per pixel; the key's depth gives the
 //    world position of the intersection.
+// Super-sampled maps (the pipeline's image-resolution render brought to the
+// latent token grid): the faces are rasterised at s times the token
+// resolution with the cameras' focal lengths and principal point scaled by
+// s, and raster_pool_kernel resolves each token's s x s pixels and pools
+// them (mean of the valid pixels' positions, foreground when at least half
+// are valid).  pool_posmaps_kernel pools maps the caller rendered itself.
 // Every decision and the position are binary32 with one rounding per
 // operation in a fixed order (explicit __f*_rn intrinsics), so the maps are
 // reproducible bit for bit.
@@ -44,18 +50,19 @@ struct Cam32 {
     float R[9], t[3], fx, fy, cx, cy;
 };
 
-// c points to global or shared memory (generic loads)
-__device__ __forceinline__ Cam32 load_cam(const geocache_camera* c) {
+// c points to global or shared memory (generic loads); the intrinsics are
+// multiplied by `scale` (binary32), the camera of an s-times finer pixel grid
+__device__ __forceinline__ Cam32 load_cam(const geocache_camera* c, float scale = 1.0f) {
     Cam32 k;
     const float* p = reinterpret_cast<const float*>(c);
 #pragma unroll
     for (int i = 0; i < 9; ++i) k.R[i] = p[i];
 #pragma unroll
     for (int i = 0; i < 3; ++i) k.t[i] = p[9 + i];
-    k.fx = p[12];
-    k.fy = p[13];
-    k.cx = p[14];
-    k.cy = p[15];
+    k.fx = __fmul_rn(p[12], scale);
+    k.fy = __fmul_rn(p[13], scale);
+    k.cx = __fmul_rn(p[14], scale);
+    k.cy = __fmul_rn(p[15], scale);
     return k;
 }
 
@@ -167,7 +174,7 @@ __device__ __forceinline__ int asset_of(const int64_t* __restrict__ face_off, in
 __global__ void __launch_bounds__(kRasterThreads, 4) raster_faces_kernel(
     const float* __restrict__ V, long long nv, const int32_t* __restrict__ F, long long nf,
     const int64_t* __restrict__ face_off, int B, const geocache_camera* __restrict__ cams, int N, int H, int W,
-    unsigned long long* __restrict__ zbuf) {
+    float scale, unsigned long long* __restrict__ zbuf) {
     __shared__ geocache_camera s_cam[GEOCACHE_MAX_VIEWS];
     __shared__ int s_asset[2];
     __shared__ FaceSlot s_slot[kRasterThreads];
@@ -204,7 +211,7 @@ __global__ void __launch_bounds__(kRasterThreads, 4) raster_faces_kernel(
     FaceSlot* slots = s_slot + (threadIdx.x & ~31);
     long long* excl_w = s_excl + (threadIdx.x & ~31);
     for (int view = 0; view < N; ++view) {
-        const Cam32 c = load_cam(b == s_asset[0] ? s_cam + view : cams + (size_t)b * N + view);
+        const Cam32 c = load_cam(b == s_asset[0] ? s_cam + view : cams + (size_t)b * N + view, scale);
         Face o;
         const bool live = ok && setup_face(c, X, H, W, o);
         const long long box = live ? (long long)(o.ihi - o.ilo + 1) * (o.jhi - o.jlo + 1) : 0;
@@ -235,11 +242,28 @@ __global__ void __launch_bounds__(kRasterThreads, 4) raster_faces_kernel(
             const int local = (int)(k - excl_w[src]);
             const int bw = q.o.ihi - q.o.ilo + 1;
             const int i = q.o.ilo + local % bw, j = q.o.jlo + local / bw;
-            const Cam32 qc = load_cam(q.b == s_asset[0] ? s_cam + view : cams + (size_t)q.b * N + view);
+            const Cam32 qc = load_cam(q.b == s_asset[0] ? s_cam + view : cams + (size_t)q.b * N + view, scale);
             const unsigned long long key = pixel_key(qc, q.o, i, j, q.f);
             if (key != kEmpty) atomicMin(zbuf + ((size_t)q.b * N + view) * (size_t)H * W + (size_t)j * W + i, key);
         }
         __syncwarp();  // the slots are rewritten for the next view
+    }
+}
+
+// World position of the surface point of pixel (i, j) whose z-buffer key is
+// `key` (not kEmpty): the ray through the pixel centre at the key's depth,
+// x_w = R^T (x_c - t).
+__device__ __forceinline__ void key_position(const Cam32& c, unsigned long long key, int i, int j, float (&X)[3]) {
+    const float s = __uint_as_float((unsigned int)(key >> 32));
+    float d0, d1;
+    ray(c, __fadd_rn((float)i, 0.5f), __fadd_rn((float)j, 0.5f), d0, d1);
+    const float xc[3] = {__fsub_rn(__fmul_rn(s, d0), c.t[0]), __fsub_rn(__fmul_rn(s, d1), c.t[1]),
+                         __fsub_rn(s, c.t[2])};
+#pragma unroll
+    for (int r = 0; r < 3; ++r) {
+        float x = __fmul_rn(c.R[r], xc[0]);
+        x = __fadd_rn(x, __fmul_rn(c.R[3 + r], xc[1]));
+        X[r] = __fadd_rn(x, __fmul_rn(c.R[6 + r], xc[2]));
     }
 }
 
@@ -254,24 +278,88 @@ __global__ void __launch_bounds__(kRasterThreads) raster_resolve_kernel(const un
         const unsigned long long key = zbuf[p];
         float X[3] = {0.0f, 0.0f, 0.0f};
         if (key != kEmpty) {
-            const Cam32 c = load_cam(cams + p / HW);  // [B, N] cameras, one per (asset, view) map
             const int pix = (int)(p % HW);
-            const float s = __uint_as_float((unsigned int)(key >> 32));
-            float d0, d1;
-            ray(c, __fadd_rn((float)(pix % W), 0.5f), __fadd_rn((float)(pix / W), 0.5f), d0, d1);
-            const float xc[3] = {__fsub_rn(__fmul_rn(s, d0), c.t[0]), __fsub_rn(__fmul_rn(s, d1), c.t[1]),
-                                 __fsub_rn(s, c.t[2])};
-#pragma unroll
-            for (int r = 0; r < 3; ++r) {
-                float x = __fmul_rn(c.R[r], xc[0]);
-                x = __fadd_rn(x, __fmul_rn(c.R[3 + r], xc[1]));
-                X[r] = __fadd_rn(x, __fmul_rn(c.R[6 + r], xc[2]));
-            }
+            key_position(load_cam(cams + p / HW), key, pix % W, pix / W, X);  // [B, N] cameras, one per map
         }
         pos[3 * p] = X[0];
         pos[3 * p + 1] = X[1];
         pos[3 * p + 2] = X[2];
         valid[p] = key != kEmpty;
+    }
+}
+
+// Token (i, j) of a token-grid map from its s x s pixels (i s + sx, j s + sy)
+// of the fine map: positions of the valid pixels summed componentwise in
+// binary32, pixel rows sy ascending and sx ascending within a row, divided
+// once by their number n; foreground when 2 n >= s * s.
+struct PoolAcc {
+    float sum[3] = {0.0f, 0.0f, 0.0f};
+    int n = 0;
+    __device__ __forceinline__ void add(const float (&X)[3]) {
+#pragma unroll
+        for (int c = 0; c < 3; ++c) sum[c] = __fadd_rn(sum[c], X[c]);
+        ++n;
+    }
+    __device__ __forceinline__ void store(int s, float* __restrict__ pos, uint8_t* __restrict__ valid, long long p) const {
+        const bool fg = n > 0 && 2 * n >= s * s;
+#pragma unroll
+        for (int c = 0; c < 3; ++c) pos[3 * p + c] = fg ? __fdiv_rn(sum[c], (float)n) : 0.0f;
+        valid[p] = fg;
+    }
+};
+
+// resolve + pool of a z-buffer rendered at s x the token grid: one thread per
+// token, grid-stride over the B * N * H * W tokens
+__global__ void __launch_bounds__(kRasterThreads) raster_pool_kernel(const unsigned long long* __restrict__ zbuf,
+                                                                      const geocache_camera* __restrict__ cams,
+                                                                      int H, int W, int s, long long n_tok,
+                                                                      float* __restrict__ pos,
+                                                                      uint8_t* __restrict__ valid) {
+    const long long HW = (long long)H * W;
+    const int Ws = W * s;
+    for (long long p = blockIdx.x * (long long)kRasterThreads + threadIdx.x; p < n_tok;
+         p += (long long)gridDim.x * kRasterThreads) {
+        const long long map = p / HW;
+        const int tok = (int)(p % HW), i = tok % W, j = tok / W;
+        const unsigned long long* zmap = zbuf + map * HW * s * s;
+        const Cam32 c = load_cam(cams + map, (float)s);
+        PoolAcc acc;
+        for (int sy = 0; sy < s; ++sy)
+            for (int sx = 0; sx < s; ++sx) {
+                const int I = i * s + sx, J = j * s + sy;
+                const unsigned long long key = __ldg(zmap + (size_t)J * Ws + I);
+                if (key == kEmpty) continue;
+                float X[3];
+                key_position(c, key, I, J, X);
+                acc.add(X);
+            }
+        acc.store(s, pos, valid, p);
+    }
+}
+
+// pool of fine maps given by the caller: pos_hi [n_maps, H s, W s, 3],
+// valid_hi [n_maps, H s, W s] -> pos [n_maps, H, W, 3], valid [n_maps, H, W]
+__global__ void __launch_bounds__(kRasterThreads) pool_posmaps_kernel(const float* __restrict__ pos_hi,
+                                                                       const uint8_t* __restrict__ valid_hi,
+                                                                       int H, int W, int s, long long n_tok,
+                                                                       float* __restrict__ pos,
+                                                                       uint8_t* __restrict__ valid) {
+    const long long HW = (long long)H * W;
+    const long long Ws = (long long)W * s;
+    for (long long p = blockIdx.x * (long long)kRasterThreads + threadIdx.x; p < n_tok;
+         p += (long long)gridDim.x * kRasterThreads) {
+        const long long map = p / HW;
+        const int tok = (int)(p % HW), i = tok % W, j = tok / W;
+        const long long base = map * HW * s * s;
+        PoolAcc acc;
+        for (int sy = 0; sy < s; ++sy)
+            for (int sx = 0; sx < s; ++sx) {
+                const long long q = base + ((long long)j * s + sy) * Ws + (long long)i * s + sx;
+                if (!__ldg(valid_hi + q)) continue;
+                const float X[3] = {__ldg(pos_hi + 3 * q), __ldg(pos_hi + 3 * q + 1), __ldg(pos_hi + 3 * q + 2)};
+                acc.add(X);
+            }
+        acc.store(s, pos, valid, p);
     }
 }
 
@@ -288,25 +376,41 @@ cudaError_t read_raster_error(unsigned int* out, bool clear, cudaStream_t s) {
     return cudaStreamSynchronize(s);
 }
 
+// grid of a grid-stride kernel over n items: at most 16 CTAs per SM
+static unsigned stride_grid(long long n) {
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const long long want = (n + kRasterThreads - 1) / kRasterThreads, cap = (long long)(sms > 0 ? sms : 1) * 16;
+    return (unsigned)(want < cap ? (want > 0 ? want : 1) : cap);
+}
+
 cudaError_t launch_raster(const float* V, long long nv, const int32_t* F, long long nf, const int64_t* face_off,
-                          int B, const geocache_camera* cams, int N, int H, int W, unsigned long long* zbuf,
+                          int B, const geocache_camera* cams, int N, int H, int W, int ss, unsigned long long* zbuf,
                           float* pos, uint8_t* valid, cudaStream_t s) {
-    const long long n_pix = (long long)B * N * H * W;
+    const long long n_tok = (long long)B * N * H * W, n_pix = n_tok * ss * ss;
     cudaError_t e = cudaMemsetAsync(zbuf, 0xff, sizeof(unsigned long long) * (size_t)n_pix, s);
     if (e != cudaSuccess) return e;
     if (nf > 0) {
         const long long gx = (nf + kRasterThreads - 1) / kRasterThreads;
         if (gx > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-        raster_faces_kernel<<<(unsigned)gx, kRasterThreads, 0, s>>>(V, nv, F, nf, face_off, B, cams, N, H, W, zbuf);
+        raster_faces_kernel<<<(unsigned)gx, kRasterThreads, 0, s>>>(V, nv, F, nf, face_off, B, cams, N, H * ss,
+                                                                    W * ss, (float)ss, zbuf);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
-    int dev = 0, sms = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const long long want = (n_pix + kRasterThreads - 1) / kRasterThreads, cap = (long long)(sms > 0 ? sms : 1) * 16;
-    raster_resolve_kernel<<<(unsigned)(want < cap ? (want > 0 ? want : 1) : cap), kRasterThreads, 0, s>>>(
-        zbuf, cams, N, H, W, n_pix, pos, valid);
+    if (ss == 1)
+        raster_resolve_kernel<<<stride_grid(n_pix), kRasterThreads, 0, s>>>(zbuf, cams, N, H, W, n_pix, pos, valid);
+    else
+        raster_pool_kernel<<<stride_grid(n_tok), kRasterThreads, 0, s>>>(zbuf, cams, H, W, ss, n_tok, pos, valid);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_pool_posmaps(const float* pos_hi, const uint8_t* valid_hi, long long n_maps, int H, int W, int ss,
+                                float* pos, uint8_t* valid, cudaStream_t s) {
+    const long long n_tok = n_maps * H * W;
+    if (n_tok == 0) return cudaSuccess;
+    pool_posmaps_kernel<<<stride_grid(n_tok), kRasterThreads, 0, s>>>(pos_hi, valid_hi, H, W, ss, n_tok, pos, valid);
     return cudaGetLastError();
 }
 

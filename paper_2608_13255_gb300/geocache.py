@@ -70,7 +70,8 @@ EXPORTS = ("geocache_build_corr", "geocache_transport_step", "geocache_reconstru
            "geocache_rotate_anchors", "geocache_device_status", "geocache_corr_record_count",
            "geocache_transport_workspace", "geocache_transport_step_noalloc", "geocache_pack_anchors",
            "geocache_unpack_anchors", "geocache_transport_step_update", "geocache_permute_records",
-           "geocache_raster_posmaps", "geocache_debug_set_wait",
+           "geocache_raster_posmaps", "geocache_debug_set_wait", "geocache_raster_posmaps_supersampled",
+           "geocache_pool_posmaps",
            "geocache_last_error", "geocache_abi_version")
 
 
@@ -101,6 +102,10 @@ def load():
         L.geocache_permute_records.restype = ctypes.c_int
         L.geocache_raster_posmaps.argtypes = [P, i64, P, i64, P, i, P, i, i, i, P, P, P, P]
         L.geocache_raster_posmaps.restype = ctypes.c_int
+        L.geocache_raster_posmaps_supersampled.argtypes = [P, i64, P, i64, P, i, P, i, i, i, i, P, P, P, P]
+        L.geocache_raster_posmaps_supersampled.restype = ctypes.c_int
+        L.geocache_pool_posmaps.argtypes = [P, P, i64, i, i, i, P, P, P]
+        L.geocache_pool_posmaps.restype = ctypes.c_int
         for name in ("geocache_pack_anchors", "geocache_unpack_anchors"):
             getattr(L, name).argtypes = [P, P, i64, i, i, P, i, P]
             getattr(L, name).restype = ctypes.c_int
@@ -335,27 +340,59 @@ def permute_records(corr: CorrHandle, perm, out=None, stream=None) -> CorrHandle
     return CorrHandle(c2, refs)
 
 
-def raster_posmaps(verts, faces, face_off, cams, H, W, zbuf=None, pos=None, valid=None, stream=None):
-    """geocache_raster_posmaps: position maps [B,N,H,W,3] f32 and validity
-    [B,N,H,W] u8 of B meshes (verts [V,3] f32, faces [F,3] i32 indexing
-    verts, face_off [B+1] i64, all on the device) seen by cams [B,N,16].
-    Returns (pos, valid); zbuf is the [B,N,H,W] int64 scratch."""
+def raster_posmaps(verts, faces, face_off, cams, H, W, zbuf=None, pos=None, valid=None, stream=None, s=1):
+    """geocache_raster_posmaps (s = 1) or geocache_raster_posmaps_supersampled
+    (rendered at s times the token grid and pooled to it): position maps
+    [B,N,H,W,3] f32 and validity [B,N,H,W] u8 of B meshes (verts [V,3] f32,
+    faces [F,3] i32 indexing verts, face_off [B+1] i64, all on the device)
+    seen by cams [B,N,16] (cameras of the H x W token grid).  Returns
+    (pos, valid); zbuf is the [B,N,s*H,s*W] int64 scratch."""
     B, N = int(cams.shape[0]), int(cams.shape[1])
     dev = cams.device
+    s = int(s)
     if zbuf is None:
-        zbuf = torch.empty((B, N, H, W), dtype=torch.int64, device=dev)
+        zbuf = torch.empty((B, N, s * H, s * W), dtype=torch.int64, device=dev)
     if pos is None:
         pos = torch.empty((B, N, H, W, 3), dtype=torch.float32, device=dev)
     if valid is None:
         valid = torch.empty((B, N, H, W), dtype=torch.uint8, device=dev)
     nv, nf = int(verts.shape[0]), int(faces.shape[0])
     n = B * N * H * W
-    _check(load().geocache_raster_posmaps(
-        _dev(verts, torch.float32, 3 * nv, "verts") if nv else None, nv,
-        _dev(faces, torch.int32, 3 * nf, "faces") if nf else None, nf,
-        _dev(face_off, torch.int64, B + 1, "face_off"), B, _dev(cams, torch.float32, 16 * B * N, "cams"), N,
-        int(H), int(W), _dev(zbuf, torch.int64, n, "zbuf"), _dev(pos, torch.float32, 3 * n, "pos"),
-        _dev(valid, torch.uint8, n, "valid"), _stream(stream)))
+    args = [_dev(verts, torch.float32, 3 * nv, "verts") if nv else None, nv,
+            _dev(faces, torch.int32, 3 * nf, "faces") if nf else None, nf,
+            _dev(face_off, torch.int64, B + 1, "face_off"), B, _dev(cams, torch.float32, 16 * B * N, "cams"), N,
+            int(H), int(W)]
+    outs = [_dev(zbuf, torch.int64, n * s * s, "zbuf"), _dev(pos, torch.float32, 3 * n, "pos"),
+            _dev(valid, torch.uint8, n, "valid"), _stream(stream)]
+    if s == 1:
+        _check(load().geocache_raster_posmaps(*args, *outs))
+    else:
+        _check(load().geocache_raster_posmaps_supersampled(*args, s, *outs))
+    return pos, valid
+
+
+def pool_posmaps(pos_hi, valid_hi, s, pos=None, valid=None, stream=None):
+    """geocache_pool_posmaps: token-grid maps ([..., H, W, 3] f32, [..., H, W]
+    u8) from maps rendered at s times the token resolution (pos_hi [..., s*H,
+    s*W, 3] f32, valid_hi [..., s*H, s*W] u8, on the device)."""
+    s = int(s)
+    Hs, Ws = int(valid_hi.shape[-2]), int(valid_hi.shape[-1])
+    if Hs % s or Ws % s:
+        raise ValueError("maps of %dx%d are not an s=%d super-sampling" % (Hs, Ws, s))
+    H, W = Hs // s, Ws // s
+    lead = tuple(valid_hi.shape[:-2])
+    n_maps = 1
+    for d in lead:
+        n_maps *= int(d)
+    if pos is None:
+        pos = torch.empty(lead + (H, W, 3), dtype=torch.float32, device=valid_hi.device)
+    if valid is None:
+        valid = torch.empty(lead + (H, W), dtype=torch.uint8, device=valid_hi.device)
+    n_hi, n = n_maps * Hs * Ws, n_maps * H * W
+    _check(load().geocache_pool_posmaps(_dev(pos_hi, torch.float32, 3 * n_hi, "pos_hi"),
+                                        _dev(valid_hi, torch.uint8, n_hi, "valid_hi"), n_maps, H, W, s,
+                                        _dev(pos, torch.float32, 3 * n, "pos"), _dev(valid, torch.uint8, n, "valid"),
+                                        _stream(stream)))
     return pos, valid
 
 

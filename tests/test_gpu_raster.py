@@ -105,3 +105,80 @@ def test_bad_face_index_is_skipped_and_reported(gc):
     ref_p, ref_v = oracle.raster_views(V, F, cams[0], H, W)
     np.testing.assert_array_equal(valid.cpu().numpy()[0], ref_v)
     np.testing.assert_array_equal(pos.cpu().numpy()[0].view(np.uint32), ref_p.view(np.uint32))
+
+
+@pytest.mark.parametrize("s,H,W", [(2, 64, 64), (4, 32, 32), (8, 16, 16), (3, 24, 40)])
+def test_supersampled_posmaps_bit_exact(gc, s, H, W):
+    # rendered at s x the token grid and pooled to it (image-resolution maps
+    # of Sec. 3.1 brought to the token grid of Sec. 3.2): validity and
+    # positions equal the oracle's render at s x with pooling, bit for bit
+    meshes, cams = _batch(H, W, synth.hunyuan_layout())
+    verts, faces, f_off, d_cams = _upload(meshes, cams)
+    pos, valid = gc.raster_posmaps(verts, faces, f_off, d_cams, H, W, s=s)
+    torch.cuda.synchronize()
+    gc.device_status()
+    pos, valid = pos.cpu().numpy(), valid.cpu().numpy()
+    for b, (V, F) in enumerate(meshes):
+        ref_p, ref_v = oracle.raster_supersampled(V, F, cams[b], H, W, s)
+        np.testing.assert_array_equal(valid[b], ref_v)
+        np.testing.assert_array_equal(pos[b].view(np.uint32), ref_p.view(np.uint32))
+    assert valid[0].mean() > 0.1 and valid[2, 0].all() and not valid[3].any()
+
+
+def test_supersampling_factor_one_is_the_plain_render(gc):
+    H, W = 48, 80
+    meshes, cams = _batch(H, W, synth.hunyuan_layout())
+    verts, faces, f_off, d_cams = _upload(meshes, cams)
+    p1, v1 = gc.raster_posmaps(verts, faces, f_off, d_cams, H, W)
+    zb = torch.empty((4, 6, H, W), dtype=torch.int64, device="cuda")
+    p2 = torch.empty_like(p1)
+    v2 = torch.empty_like(v1)
+    gc.load().geocache_raster_posmaps_supersampled(
+        verts.data_ptr(), verts.shape[0], faces.data_ptr(), faces.shape[0], f_off.data_ptr(), 4, d_cams.data_ptr(), 6,
+        H, W, 1, zb.data_ptr(), p2.data_ptr(), v2.data_ptr(), None)
+    torch.cuda.synchronize()
+    assert torch.equal(v1, v2) and torch.equal(p1.view(torch.int32), p2.view(torch.int32))
+
+
+@pytest.mark.parametrize("s,H,W", [(8, 32, 32), (3, 37, 53), (1, 16, 24)])
+def test_pool_posmaps_bit_exact(gc, s, H, W):
+    # caller-rendered fine maps pooled on the GPU: equal to the oracle's
+    # pooling bit for bit (maps rendered by the oracle at s x, several views)
+    meshes, cams = _batch(H, W, synth.hunyuan_layout())
+    fine_p, fine_v = oracle.raster_views(*meshes[0], oracle.scaled_camera(cams[0], s), H * s, W * s)
+    ref_p, ref_v = oracle.pool(fine_p, fine_v, s)
+    pos, valid = gc.pool_posmaps(torch.from_numpy(fine_p).cuda(), torch.from_numpy(fine_v).cuda(), s)
+    torch.cuda.synchronize()
+    gc.device_status()
+    np.testing.assert_array_equal(valid.cpu().numpy(), ref_v)
+    np.testing.assert_array_equal(pos.cpu().numpy().view(np.uint32), ref_p.view(np.uint32))
+    assert ref_v.mean() > 0.05
+
+
+def test_supersampled_posmaps_feed_the_correspondence_build(gc):
+    # pooled maps (s = 4) into geocache_build_corr: tau, keep masks, tables
+    # and records bit-exact against the oracle built on the oracle's pooled maps
+    H = W = 64
+    s = 4
+    meshes, cams = _batch(H, W, synth.hunyuan_layout())
+    verts, faces, f_off, d_cams = _upload(meshes[:1], cams[:1])
+    pos, valid = gc.raster_posmaps(verts, faces, f_off, d_cams, H, W, s=s)
+    ref_p, ref_v = oracle.raster_supersampled(*meshes[0], cams[0], H, W, s)
+    np.testing.assert_array_equal(valid.cpu().numpy()[0], ref_v)
+    corr = gc.build_sparse_corr(pos, valid, d_cams, K=4, tables=True)
+    torch.cuda.synchronize()
+    gc.device_status()
+    tau_ref = oracle.tau(ref_p[None], ref_v[None])
+    np.testing.assert_array_equal(corr.tau.cpu().numpy(), tau_ref)
+    idx, w, band = oracle.build_corr(ref_p[None], ref_v[None], cams[:1], tau_ref, K=4)
+    inband = np.broadcast_to(band[..., None] > 0, idx.shape)
+    assert not ((corr.idx.cpu().numpy() != idx) & ~inband).any()
+    assert (idx >= 0).any(-1).mean() > 0.01
+
+
+def test_supersampled_sizes_are_checked(gc):
+    meshes, cams = _batch(16, 16, synth.hunyuan_layout())
+    verts, faces, f_off, d_cams = _upload(meshes[:1], cams[:1])
+    with pytest.raises(gc.GeocacheError) as ei:
+        gc.raster_posmaps(verts, faces, f_off, d_cams, 16, 16, s=17)
+    assert ei.value.status == gc.ESHAPE
