@@ -50,6 +50,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--no-raster", action="store_true", help="skip the position-map rasteriser measurement")
+    p.add_argument("--no-workloads", action="store_true",
+                   help="skip the other workloads' cached-step measurements (ring12_128, per-asset latency)")
     p.add_argument("--cpu-assets", type=int, default=32,
                    help="assets in the oracle's timed sample for cpu_baseline (one trajectory, ~10-30 s)")
     p.add_argument("--ref-assets", type=int, default=2,
@@ -83,10 +85,10 @@ def dist_env():
 
 
 def workload(args, rank=0):
+    """This rank's shard of the job's assets: global assets rank*B .. rank*B + B - 1
+    (B = --assets per GPU; weak scaling), each rendered from its own seed."""
     from paper_2608_13255_gb300 import synth
-    # each rank renders its own independent assets
-    base = synth.WORKLOADS[args.workload]
-    return synth.make_workload(args.workload, B=args.assets, seed=base["seed"] + 7919 * rank)
+    return synth.make_workload(args.workload, B=args.assets, first_asset=rank * args.assets)
 
 
 def describe(w):
@@ -235,6 +237,88 @@ def measure_sweep(traj, sizes, reps=24):
     return out
 
 
+def time_cached_steps(w, B, dev, reps=24, seed=3):
+    """One graph of `reps` cached transport steps of workload w replicated to
+    B assets (its own correspondence build, sparse mode), the anchor set
+    rotating as the workload's schedule rotates it over its cached steps and
+    the x0 cache ping-ponging between two buffers; latents in place.
+    Returns (us per step, algorithmic bytes per step, target view-pixels per step)."""
+    import torch
+    from paper_2608_13255_gb300 import geocache as gc
+    from paper_2608_13255_gb300 import synth
+    wb = synth.replicate_assets(w, B)
+    pos, valid, cams = (torch.from_numpy(a).to(dev) for a in (wb.pos, wb.valid, wb.cams))
+    corr = gc.build_sparse_corr(pos, valid, cams, K=wb.K, tol_frac=wb.tol_frac)
+    wsp = torch.empty(max(corr.workspace_floats(wb.C), 4), dtype=torch.float32, device=dev)
+    cached = [t for t in range(wb.S) if not gc.rotate_anchors(wb.N, wb.a, t, wb.S, wb.schedule)[1]]
+    sets = []
+    for t in cached:
+        a = tuple(gc.rotate_anchors(wb.N, wb.a, t, wb.S, wb.schedule)[0])
+        if a not in sets:
+            sets.append(a)
+    g0 = torch.Generator(device=dev).manual_seed(seed)
+    shp = (B, wb.N, wb.C, wb.H, wb.W)
+    bufs = [torch.randn(shp, device=dev, generator=g0) for _ in range(2)]
+    lat = torch.bfloat16 if wb.dtype == "bf16" else torch.float32
+    x = torch.randn(shp, device=dev, generator=g0).to(lat)
+    new = {a: torch.randn((B, wb.a, wb.C, wb.H, wb.W), device=dev, generator=g0) for a in sets}
+    p = synth.recon_params(wb, cached[0])
+    r = gc.make_recon(p["sampler"], a_t=p.get("a_t", 0), a_prev=p.get("a_prev", 0), sigma=p.get("sigma", 0),
+                      sigma_next=p.get("sigma_next", 0))
+
+    def one(i):
+        a = sets[i % len(sets)]
+        gc.transport_step(corr, list(a), wb.C, new[a], bufs[i % 2], bufs[(i + 1) % 2], x, x, r, workspace=wsp)
+    for i in range(2):
+        one(i)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for i in range(reps):
+            one(i)
+    g.replay()
+    ts = []
+    for _ in range(3):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1) * 1e3 / reps)
+    gc.device_status()
+    us = statistics.median(ts)
+    return us, step_bytes(wb), B * (wb.N - wb.a) * wb.H * wb.W, sets
+
+
+def measure_workloads(dev, reps=24):
+    """Cached-step times of the other workloads (sparse mode, 24-step graphs,
+    anchors rotating as each workload's schedule rotates them):
+    * ring12_128 (12 views, 128 x 128 x 16 bf16, 4 anchors, FM-Euler)
+      replicated to 8 assets (335 MB per step, more than the L2): a DRAM
+      figure against the measured copy peak;
+    * the paper's per-asset regime, one asset per step (hunyuan64,
+      solids96, ring12_128) and batch128 at its base batch of 8 assets:
+      these steps fit in the 129 MB L2, so they are reported as latency."""
+    from paper_2608_13255_gb300 import synth
+    peak = measured_peak()[0]
+    out = {}
+    r12 = synth.make_workload("ring12_128")
+    for name, w, B in (("ring12_128_x8", r12, 8), ("ring12_128_x1", r12, 1),
+                       ("hunyuan64_x1", synth.make_workload("hunyuan64"), 1),
+                       ("solids96_x1", synth.make_workload("solids96"), 1),
+                       ("batch128_x8", synth.make_workload("batch128", B=8), 8)):
+        us, nbytes, pix, sets = time_cached_steps(w, B, dev, reps)
+        d = {"us_per_step": us, "alg_bytes": nbytes, "target_pixels_per_s": pix / us * 1e6,
+             "anchor_sets": [list(a) for a in sets]}
+        if nbytes > L2_BYTES:
+            d["frac_of_peak"] = nbytes / us / 1e3 / peak
+        else:
+            d["fits_in_l2"] = True
+        out[name] = d
+    out["what"] = ("one cached step (sparse mode) per graph node, %d steps per graph, median of 3 replays; "
+                   "frac_of_peak only where a step moves more than the L2 holds" % reps)
+    return out
+
+
 def measure_raster(dev, B, N_layout, H, W, reps=10, cpu_assets=2):
     """Position maps of B meshes (icosphere subdivision 6 with smooth radial
     noise: 40962 vertices, 81920 faces; four distinct meshes tiled over the
@@ -280,6 +364,62 @@ def measure_raster(dev, B, N_layout, H, W, reps=10, cpu_assets=2):
             "covered_frac": float(valid.float().mean()), "launches_per_call": 2,
             "cpu_oracle": {"pixels_per_s": cpu_assets * N * H * W / cpu_s, "cores": 1,
                            "sample": "%d of the meshes, all views" % cpu_assets}}
+
+
+def measure_supersampled(dev, B=16, H=128, W=128, s=4, reps=5):
+    """Position maps rendered at s times the token grid and pooled to it
+    (geocache_raster_posmaps_supersampled: the image-resolution render of a
+    pipeline, 512 x 512 for 128 x 128 tokens at s = 4), and the pooling alone
+    of caller-rendered fine maps (geocache_pool_posmaps, HBM-bound: 13 B read
+    per fine pixel, 13 B written per token).  B meshes of the rasteriser
+    measurement, the workload's 6 cameras."""
+    import torch
+    from paper_2608_13255_gb300 import geocache as gc
+    from paper_2608_13255_gb300 import synth
+    base = [synth.blob_mesh(6, 0.15, np.random.default_rng(100 + k)) for k in range(4)]
+    meshes = [(base[b % 4][0].astype(np.float32), base[b % 4][1].astype(np.int32)) for b in range(B)]
+    layout = synth.hunyuan_layout()
+    cams = np.stack([np.stack([synth.look_at_camera(az + 7.0 * b, el, H, W) for az, el in layout]) for b in range(B)])
+    v_off = np.cumsum([0] + [len(V) for V, _ in meshes])
+    f_off = torch.from_numpy(np.cumsum([0] + [len(F) for _, F in meshes]).astype(np.int64)).to(dev)
+    verts = torch.from_numpy(np.concatenate([V for V, _ in meshes])).to(dev)
+    faces = torch.from_numpy(np.concatenate([F + v_off[b] for b, (_, F) in enumerate(meshes)]).astype(np.int32)).to(dev)
+    d_cams = torch.from_numpy(cams).to(dev)
+    N = len(layout)
+    zbuf = torch.empty((B, N, s * H, s * W), dtype=torch.int64, device=dev)
+    pos = torch.empty((B, N, H, W, 3), dtype=torch.float32, device=dev)
+    valid = torch.empty((B, N, H, W), dtype=torch.uint8, device=dev)
+
+    def timed(fn):
+        fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for _ in range(reps):
+            fn()
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / reps
+    us_ss = timed(lambda: gc.raster_posmaps(verts, faces, f_off, d_cams, H, W, zbuf, pos, valid, s=s))
+    # fine maps rendered directly at s x (cameras scaled), then pooled
+    cams_hi = d_cams.clone()
+    cams_hi[..., 12:16] *= s
+    fine_p = torch.empty((B, N, s * H, s * W, 3), dtype=torch.float32, device=dev)
+    fine_v = torch.empty((B, N, s * H, s * W), dtype=torch.uint8, device=dev)
+    gc.raster_posmaps(verts, faces, f_off, cams_hi, s * H, s * W, zbuf, fine_p, fine_v)
+    pos2, valid2 = torch.empty_like(pos), torch.empty_like(valid)
+    us_pool = timed(lambda: gc.pool_posmaps(fine_p, fine_v, s, pos2, valid2))
+    torch.cuda.synchronize()
+    gc.device_status()
+    same = bool(torch.equal(valid, valid2) and torch.equal(pos.view(torch.int32), pos2.view(torch.int32)))
+    fine_px = B * N * s * s * H * W
+    pool_bytes = fine_px * 13 + B * N * H * W * 13
+    return {"what": "%d meshes x %d views, %dx%d tokens rendered at %dx%d (s = %d), 81920 faces each"
+                    % (B, N, H, W, s * H, s * W, s),
+            "raster_supersampled_us": us_ss, "fine_pixels_per_s": fine_px / us_ss * 1e6,
+            "pool_us": us_pool, "pool_alg_bytes": pool_bytes, "pool_GBs": pool_bytes / us_pool / 1e3,
+            "pool_frac_of_peak": pool_bytes / us_pool / 1e3 / measured_peak()[0],
+            "pooled_equals_fused": same}
 
 
 class Trajectory:
@@ -566,9 +706,10 @@ def measured_peak():
 
 
 # ------------------------------------------------------------ CPU oracle --
-def oracle_trajectory(w, steps=None):
+def oracle_trajectory(w, steps=None, state=False):
     """The CPU oracle, as it stands, over one trajectory of workload w.
-    Returns (cached target view-pixels processed, seconds)."""
+    Returns (cached target view-pixels processed, seconds), plus the final
+    latents and x0 cache when state is true."""
     import oracle
     from paper_2608_13255_gb300 import synth
     t0 = time.perf_counter()
@@ -593,6 +734,8 @@ def oracle_trajectory(w, steps=None):
             pixels += w.B * (w.N - w.a) * w.H * w.W
         if w.dtype == "bf16":
             x = (oracle.round_bf16(x).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    if state:
+        return pixels, time.perf_counter() - t0, x, cache
     return pixels, time.perf_counter() - t0
 
 
@@ -606,9 +749,12 @@ def cpu_baseline(args, w_full):
 
 
 def _asset_subset(w, idx):
-    """Workload w restricted to the assets idx (same recipe, fewer assets)."""
+    """Workload w restricted to the contiguous assets idx (same recipe, fewer assets)."""
+    idx = np.asarray(idx)
+    assert len(idx) and (np.diff(idx) == 1).all(), "asset subsets are contiguous ranges"
     out = type(w)(**{**w.__dict__})
     out.B = len(idx)
+    out.first_asset = w.first_asset + int(idx[0])
     out.cams = np.ascontiguousarray(w.cams[idx])
     out.pos = np.ascontiguousarray(w.pos[idx])
     out.valid = np.ascontiguousarray(w.valid[idx])
@@ -797,11 +943,13 @@ def main():
     if rank == 0 and args.corr == "sparse" and use_graphs and args.sweep:
         sweep = measure_sweep(traj, [int(x) for x in args.sweep.split(",")])
     stages = measure_stages(traj) if rank == 0 and use_graphs else None
+    workloads = measure_workloads(dev) if rank == 0 and use_graphs and not args.no_workloads else None
     raster = None
     if rank == 0 and not args.no_raster:
         from paper_2608_13255_gb300 import synth
         layout = synth.hunyuan_layout() if w.N == 6 else synth.ring8_polar4_layout()[:w.N]
         raster = measure_raster(dev, w.B, layout, w.H, w.W)
+        raster["supersampled"] = measure_supersampled(dev)
 
     e2e = None
     if not args.no_e2e:
@@ -839,6 +987,7 @@ def main():
         "stages": stages,
         "ablations": ablations,
         "batch_sweep": sweep,
+        "workloads": workloads,
         "raster_posmaps": raster,
         "clocks": clocks.summary(),
         "e2e": e2e,

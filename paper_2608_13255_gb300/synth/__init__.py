@@ -350,6 +350,7 @@ class Workload:
     mesh: str             # "sphere" | "blob2562" | "solids" | "blob40962" | "mixed"
     seed: int
     tol_frac: float = 0.01
+    first_asset: int = 0        # global index of asset 0 (a shard of a larger batch starts there)
     cams: np.ndarray = None     # [B,N,16] f32
     pos: np.ndarray = None      # [B,N,H,W,3] f32
     valid: np.ndarray = None    # [B,N,H,W] u8
@@ -410,6 +411,8 @@ WORKLOADS = {
 
 
 def asset_seed(w_seed: int, asset: int, B: int) -> int:
+    """Seed of the geometry of the asset with global index `asset` in a batch
+    of B (a single-asset workload uses the workload seed itself)."""
     return w_seed if B == 1 else w_seed * 1000 + asset
 
 
@@ -425,13 +428,15 @@ def make_workload(name: str, **overrides) -> Workload:
     w.pos = np.zeros((w.B, w.N, w.H, w.W, 3), np.float32)
     w.valid = np.zeros((w.B, w.N, w.H, w.W), np.uint8)
     cache = {}
+    single = w.B == 1 and w.first_asset == 0
     for b in range(w.B):
-        s = asset_seed(w.seed, b, w.B)
+        g = w.first_asset + b  # global asset index
+        s = asset_seed(w.seed, g, 1 if single else 2)
         # assets of the same mesh kind and seed render identically; cache by seed
-        key = (w.mesh, s, b % 3 if w.mesh == "mixed" else 0)
+        key = (w.mesh, s, g % 3 if w.mesh == "mixed" else 0)
         if key not in cache:
             rng = np.random.default_rng(s)
-            shape = _shape_for(w.mesh, rng, b)
+            shape = _shape_for(w.mesh, rng, g)
             cache[key] = render_asset(shape, w.cams[b], w.H, w.W)
         w.pos[b], w.valid[b] = cache[key]
     return w
@@ -457,19 +462,28 @@ def _rng(*key) -> np.random.Generator:
 
 
 def initial_latents(w: Workload):
-    """x_T ~ N(0,1) and x0 at step 0 ~ N(0,1), shape [B,N,C,H,W] float32."""
-    shp = (w.B, w.N, w.C, w.H, w.W)
-    xT = _rng(w.seed, 0xA11CE).standard_normal(shp, dtype=np.float32)
-    x0 = _rng(w.seed, 0x0B0B0).standard_normal(shp, dtype=np.float32)
+    """x_T ~ N(0,1) and x0 at step 0 ~ N(0,1), shape [B,N,C,H,W] float32.
+    Each asset draws from its own stream, keyed by its global index, so a
+    shard of a batch gets the same values as the whole batch."""
+    shp = (w.N, w.C, w.H, w.W)
+    xT = np.empty((w.B,) + shp, np.float32)
+    x0 = np.empty((w.B,) + shp, np.float32)
+    for b in range(w.B):
+        g = w.first_asset + b
+        xT[b] = _rng(w.seed, 0xA11CE, g).standard_normal(shp, dtype=np.float32)
+        x0[b] = _rng(w.seed, 0x0B0B0, g).standard_normal(shp, dtype=np.float32)
     return xT, x0
 
 
 def delta(w: Workload, step: int, views, std: float = 0.1) -> np.ndarray:
-    """Per-step synthetic x0 update for the given views: [B,len(views),C,H,W]."""
+    """Per-step synthetic x0 update for the given views: [B,len(views),C,H,W]
+    (one stream per step, view and global asset index)."""
     out = np.empty((w.B, len(views), w.C, w.H, w.W), np.float32)
-    for j, v in enumerate(views):
-        out[:, j] = _rng(w.seed, 0xDE17A, step, v).standard_normal(
-            (w.B, w.C, w.H, w.W), dtype=np.float32) * np.float32(std)
+    for b in range(w.B):
+        g = w.first_asset + b
+        for j, v in enumerate(views):
+            out[b, j] = _rng(w.seed, 0xDE17A, step, v, g).standard_normal(
+                (w.C, w.H, w.W), dtype=np.float32) * np.float32(std)
     return out
 
 
