@@ -248,7 +248,7 @@ def time_cached_steps(w, B, dev, reps=24, seed=3):
     from paper_2608_13255_gb300 import synth
     wb = synth.replicate_assets(w, B)
     pos, valid, cams = (torch.from_numpy(a).to(dev) for a in (wb.pos, wb.valid, wb.cams))
-    corr = gc.build_sparse_corr(pos, valid, cams, K=wb.K, tol_frac=wb.tol_frac)
+    corr = gc.build_sparse_corr(pos, valid, cams, K=wb.K, tol_frac=wb.tol_frac, source_index=wb.C >= 8)
     wsp = torch.empty(max(corr.workspace_floats(wb.C), 4), dtype=torch.float32, device=dev)
     cached = [t for t in range(wb.S) if not gc.rotate_anchors(wb.N, wb.a, t, wb.S, wb.schedule)[1]]
     sets = []

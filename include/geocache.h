@@ -29,7 +29,7 @@
 extern "C" {
 #endif
 
-#define GEOCACHE_ABI_VERSION 1
+#define GEOCACHE_ABI_VERSION 2
 #define GEOCACHE_MAX_VIEWS 64   /* N <= 64 */
 #define GEOCACHE_MAX_CHANNELS 1024
 #define GEOCACHE_TILE_TOKENS 1024 /* tokens per tile of the sparse operator (row-major token order) */
@@ -122,6 +122,14 @@ typedef struct {
     geocache_tap_record* records;   /* device [max_records], sorted by (b, v, u, token); or NULL */
     int64_t max_records;            /* capacity of records */
     geocache_corr_mode mode;        /* taps used by geocache_transport_step */
+    int32_t* src_ptr;               /* device [B*N*T + 1] i32 or NULL: source index of the records (with
+                                       src_rec; needs records).  Group g = (b*N + u)*T + st holds the records
+                                       of source view u of asset b whose first kept tap lies in tile st:
+                                       entries [g ? src_ptr[g-1] : 0, src_ptr[g]) of src_rec.  Sparse steps
+                                       with C >= 8 then apply the records per source tile (same results). */
+    int32_t* src_rec;               /* device [max_records][2] i32, 8-byte aligned, or NULL: entries
+                                       (record index, target view v); their order within a group is not
+                                       specified */
 } geocache_corr;
 
 /* Sampler step parameters (Sec. 3.2, closed-form conversion after Eq. 1).
@@ -168,8 +176,9 @@ typedef struct {
  * every ordered pair (v, u), the tables idx/w (when both are non-NULL) and
  * the keep masks (when keep is non-NULL): the diagonal u == v and
  * background targets hold idx -1 / w 0 / keep 0.  When tile_ptr is given
- * (it needs keep) the tile offsets of the sparse form are written, and when
- * records is also given the records are written.  The call is asynchronous;
+ * (it needs keep) the tile offsets of the sparse form are written, when
+ * records is also given the records are written, and when src_ptr and
+ * src_rec are also given the source index is written.  The call is asynchronous;
  * size records with geocache_corr_record_count (the count depends only on
  * the geometry).  Records beyond max_records are dropped and flagged in the
  * device status word (geocache_device_status then returns ESHAPE).

@@ -179,6 +179,20 @@ int geocache_build_corr(geocache_corr* c, void* stream) {
     if (c->records && (overlap(c->records, (size_t)c->max_records * 16, c->pos, texels * 12) ||
                        overlap(c->records, (size_t)c->max_records * 16, c->keep, texels * c->N)))
         return fail(GEOCACHE_EALIAS, "records overlap another buffer");
+    if ((c->src_ptr == nullptr) != (c->src_rec == nullptr))
+        return fail(GEOCACHE_EINVAL, "src_ptr and src_rec must both be given or both NULL");
+    if (c->src_ptr) {
+        if (!c->records) return fail(GEOCACHE_EINVAL, "the source index needs records");
+        if ((uintptr_t)c->src_rec & 7) return fail(GEOCACHE_EINVAL, "src_rec must be 8-byte aligned");
+        const size_t ng = ((size_t)c->B * c->N * geocache::tiles_per_view(c->H, c->W) + 1) * 4;
+        const size_t nr = (size_t)c->max_records * 8, nt = ((size_t)c->B * c->N * c->N * geocache::tiles_per_view(c->H, c->W) + 1) * 4;
+        const void* bufs[4] = {c->records, c->tile_ptr, c->keep, c->pos};
+        const size_t sizes[4] = {(size_t)c->max_records * 16, nt, texels * c->N, texels * 12};
+        if (overlap(c->src_ptr, ng, c->src_rec, nr)) return fail(GEOCACHE_EALIAS, "src_ptr and src_rec overlap");
+        for (int i = 0; i < 4; ++i)
+            if (overlap(c->src_ptr, ng, bufs[i], sizes[i]) || overlap(c->src_rec, nr, bufs[i], sizes[i]))
+                return fail(GEOCACHE_EALIAS, "the source index overlaps another buffer");
+    }
     cudaStream_t s = (cudaStream_t)stream;
     cudaError_t e = geocache::launch_tau(c->pos, c->valid, c->B, c->N, c->H, c->W, c->tol_frac, c->tau, s);
     if (e != cudaSuccess) return cuda_fail(e, "tau kernel launch");
@@ -194,6 +208,10 @@ int geocache_build_corr(geocache_corr* c, void* stream) {
         e = geocache::launch_fill_records(*c, s);
         if (e != cudaSuccess) return cuda_fail(e, "record kernel launch");
     }
+    if (c->src_ptr) {
+        e = geocache::launch_src_index(*c, s);
+        if (e != cudaSuccess) return cuda_fail(e, "source index kernel launch");
+    }
     return ok();
 }
 
@@ -202,6 +220,8 @@ int geocache_corr_record_count(geocache_corr* c, int64_t* count, void* stream) {
     if (!c->keep || !c->tile_ptr) return fail(GEOCACHE_EINVAL, "counting records needs keep and tile_ptr");
     geocache_corr d = *c;
     d.records = nullptr;
+    d.src_ptr = nullptr;
+    d.src_rec = nullptr;
     d.idx = nullptr;
     d.w = nullptr;
     int st = geocache_build_corr(&d, stream);
@@ -302,6 +322,8 @@ int geocache_transport_step_update(const geocache_corr* c, geocache_update updat
     t.tile_ptr = c->tile_ptr;
     t.records = c->records;
     t.max_records = c->max_records;
+    t.src_ptr = c->mode == GEOCACHE_CORR_SPARSE ? c->src_ptr : nullptr;
+    t.src_rec = c->mode == GEOCACHE_CORR_SPARSE ? c->src_rec : nullptr;
     t.workspace = workspace;
     t.x0_new = x0_anchor_new; t.x0_prev = x0_prev; t.x0_out = x0_out;
     t.x_t = x_t; t.x_next = x_next; t.pred_out = recon ? recon->pred_out : nullptr;

@@ -38,6 +38,8 @@ struct TransportArgs {
     const int32_t* tile_ptr;
     const geocache_tap_record* records;
     long long max_records;
+    const int32_t* src_ptr;             // source index of the records (optional; see geocache_corr)
+    const int32_t* src_rec;
     float* workspace;
     const float* x0_new;
     const float* x0_prev;
@@ -63,6 +65,8 @@ cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s);
 // tile_ptr (tile_ptr[n] = total, or -1 when the total exceeds INT32_MAX)
 cudaError_t launch_tile_ptr(const geocache_corr& c, cudaStream_t s);
 cudaError_t launch_fill_records(const geocache_corr& c, cudaStream_t s);
+// source index of the records (c.src_ptr, c.src_rec), after the records
+cudaError_t launch_src_index(const geocache_corr& c, cudaStream_t s);
 cudaError_t launch_permute_records(const geocache_tap_record* src, const int32_t* perm, geocache_tap_record* dst,
                                    long long n, cudaStream_t s);
 __host__ __device__ int tiles_per_view(int H, int W);

@@ -53,7 +53,9 @@ __device__ __forceinline__ float tap_term(bool copy, float w, float xn, float xp
 // n covering anchors' terms: x0 + g/n (Eq. 1, normalised multi-anchor sum),
 // or g/n under the value copy.
 __device__ __forceinline__ float fold_one(bool copy, float x0, float g, int n) {
-    const float m = n == 1 ? g : __fdiv_rn(g, (float)n);
+    // g / n correctly rounded; for n a power of two that is exactly g * (1 / n)
+    const float m = n == 1 ? g
+                           : ((n & (n - 1)) == 0 ? __fmul_rn(g, __frcp_rn((float)n)) : __fdiv_rn(g, (float)n));
     return copy ? m : __fadd_rn(x0, m);
 }
 
@@ -500,6 +502,63 @@ cudaError_t launch_fill_records(const geocache_corr& c, cudaStream_t s) {
     else
         fill_records_kernel<1><<<grid, 256, 0, s>>>(c.pos, c.cams, c.keep, c.tile_ptr, c.N, c.H, c.W, T, c.records,
                                                     c.max_records);
+    return cudaGetLastError();
+}
+
+// Source index of the sparse form: the records grouped by (asset b, source
+// view u, source tile st), st = the tile of the record's first kept tap, so
+// that a step can apply the records per source tile with the anchor's tile
+// staged in shared memory.  Entries are (record index, target view).  Two
+// passes over the records: a count per group, then (after the exclusive scan
+// of the counts into src_ptr) a scatter that advances src_ptr[g] by one per
+// entry, which leaves src_ptr[g] = the end of group g (its start is
+// src_ptr[g - 1], 0 for g = 0).  The order within a group is that of the
+// atomics; nothing depends on it (each record's increment is computed on its
+// own).
+template <int K>
+__device__ __forceinline__ int first_kept_tap(int mask, int q_tl, int W) {
+    if (K == 1) return q_tl;
+    const int k = __ffs(mask) - 1;  // the lowest kept tap: TL, TR, BL, BR
+    return q_tl + (k & 1) + (k >> 1) * W;
+}
+
+template <int K, bool SCATTER>
+__global__ void __launch_bounds__(256) src_index_kernel(const int32_t* __restrict__ tile_ptr,
+                                                        const geocache_tap_record* __restrict__ rec,
+                                                        long long max_records, int N, int W, int T,
+                                                        int32_t* __restrict__ src_ptr, int2* __restrict__ src_rec) {
+    const int tile = blockIdx.x, vu = blockIdx.y, b = blockIdx.z;
+    const int v = vu / N, u = vu % N;
+    if (u == v) return;
+    const size_t ti = ((size_t)b * N * N + vu) * T + tile;
+    const long long x0 = __ldg(tile_ptr + ti), x1 = __ldg(tile_ptr + ti + 1);
+    const int r0 = (int)(x0 < 0 ? 0 : (x0 < max_records ? x0 : max_records));
+    const int r1 = (int)(x1 < 0 ? 0 : (x1 < max_records ? x1 : max_records));
+    for (int r = r0 + threadIdx.x; r < r1; r += 256) {
+        const int4 x = __ldg(reinterpret_cast<const int4*>(rec) + r);
+        const int q = first_kept_tap<K>((int)((uint32_t)x.x >> 28), x.y, W);
+        const size_t g = ((size_t)b * N + u) * T + q / GEOCACHE_TILE_TOKENS;
+        if (!SCATTER) atomicAdd(src_ptr + g, 1);
+        else src_rec[atomicAdd(src_ptr + g, 1)] = make_int2(r, v);
+    }
+}
+
+cudaError_t launch_src_index(const geocache_corr& c, cudaStream_t s) {
+    const int T = tiles_per_view(c.H, c.W);
+    const long long groups = (long long)c.B * c.N * T;
+    cudaError_t e = cudaMemsetAsync(c.src_ptr, 0, (groups + 1) * sizeof(int32_t), s);
+    if (e != cudaSuccess) return e;
+    const dim3 grid(T, c.N * c.N, c.B);
+    int2* out = reinterpret_cast<int2*>(c.src_rec);
+    if (c.K == 4)
+        src_index_kernel<4, false><<<grid, 256, 0, s>>>(c.tile_ptr, c.records, c.max_records, c.N, c.W, T, c.src_ptr, out);
+    else
+        src_index_kernel<1, false><<<grid, 256, 0, s>>>(c.tile_ptr, c.records, c.max_records, c.N, c.W, T, c.src_ptr, out);
+    exclusive_scan_kernel<<<1, 1024, 0, s>>>(c.src_ptr, groups);
+    if (c.K == 4)
+        src_index_kernel<4, true><<<grid, 256, 0, s>>>(c.tile_ptr, c.records, c.max_records, c.N, c.W, T, c.src_ptr, out);
+    else
+        src_index_kernel<1, true><<<grid, 256, 0, s>>>(c.tile_ptr, c.records, c.max_records, c.N, c.W, T, c.src_ptr, out);
     return cudaGetLastError();
 }
 
@@ -1187,10 +1246,11 @@ __device__ __forceinline__ int record_offset(const int32_t* __restrict__ tile_pt
     return (int)(x < 0 ? 0 : (x < cap ? x : cap));
 }
 
-// Records of one pair applied by one CTA slice (grid-stride over the pair's records).
-// COPY: the value-copy ablation (no x0(t-1) gathers).
+// Records of one pair applied by one CTA slice (grid-stride over the pair's
+// records), channels [cg, cg + 4).  COPY: the value-copy ablation (no x0(t-1)
+// gathers).
 template <int K, bool COPY>
-__device__ __forceinline__ void apply_records(const TransportArgs& args, int pair_id, int slice, int n_slices) {
+__device__ __forceinline__ void apply_records(const TransportArgs& args, int pair_id, int slice, int n_slices, int cg) {
     const int N = args.N, C = args.C, a = args.a;
     const int HW = args.H * args.W;
     const int T = tiles_per_view_dev(args.H, args.W);
@@ -1212,7 +1272,7 @@ __device__ __forceinline__ void apply_records(const TransportArgs& args, int pai
         taps_from_record<K>((int)((uint32_t)rec.x >> 28), rec.y, __int_as_float(rec.z), __int_as_float(rec.w),
                             args.W, tp);
         float* out = args.workspace + (size_t)r * C;
-        for (int cg = 0; cg < C; cg += 4) {
+        {
             const int cn = C - cg < 4 ? C - cg : 4;
             float dn[K][4], dp[K][4];
 #pragma unroll
@@ -1248,7 +1308,8 @@ __device__ __forceinline__ void apply_records(const TransportArgs& args, int pai
 }
 
 // Phase A: n_apply record-slice CTAs and n_stream anchor-view CTAs (tiles of
-// kTileTokens tokens), interleaved evenly in block order.
+// kTileTokens tokens), each for one group of 4 channels, interleaved evenly in
+// block order.
 // Resident CTAs per SM the phases are compiled for, by latent type: with
 // bf16 latents 6 (phase A, at most 40 registers) and 5 (phase B) put more
 // gathers and streamed rows in flight than the few spilled registers cost
@@ -1261,7 +1322,7 @@ constexpr int kPhaseBBlocks = sizeof(T) == 2 ? 5 : 1;
 
 template <typename T, int K, bool VEC, bool COPY>
 __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_kernel(const TransportArgs args, int n_apply,
-                                                                  int n_stream, int n_slices) {
+                                                                  int n_stream, int n_slices, int n_cg) {
     pdl_launch_dependents();
     const long long total = (long long)n_apply + n_stream;
     const long long k = blockIdx.x;
@@ -1269,39 +1330,41 @@ __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_ker
     const bool is_stream = (int)((k + 1) * n_stream / total) > s_before;
     if (!is_stream) {
         const int ai = (int)k - s_before;
-        apply_records<K, COPY>(args, ai / n_slices, ai % n_slices, n_slices);
+        const int aj = ai / n_cg;
+        apply_records<K, COPY>(args, aj / n_slices, aj % n_slices, n_slices, (ai % n_cg) * 4);
         return;
     }
     const int n_tiles = tiles_per_view_dev(args.H, args.W);
-    const int tile = s_before % n_tiles;
-    const int slot = (s_before / n_tiles) % args.a;
-    const int b = s_before / (n_tiles * args.a);
+    const int cg = (s_before % n_cg) * 4;
+    const int tile = (s_before / n_cg) % n_tiles;
+    const int slot = (s_before / (n_cg * n_tiles)) % args.a;
+    const int b = s_before / (n_cg * n_tiles * args.a);
     const int v = args.anchors[slot];
     const int HW = args.H * args.W;
     const int tile0 = tile * kTileTokens;
     const int p0 = tile0 + 4 * threadIdx.x;
     if (p0 >= HW) return;
     const int cnt = HW - p0 < 4 ? HW - p0 : 4;
-    for (int cg = 0; cg < args.C; cg += 4) {
-        const int cn = args.C - cg < 4 ? args.C - cg : 4;
-        QuadRows<T, VEC> q;
-        q.load(args, b, v, slot, p0, cnt, cg, cn);
-        q.store(args, b, v, p0, cnt, cg, cn);
-    }
+    const int cn = args.C - cg < 4 ? args.C - cg : 4;
+    QuadRows<T, VEC> q;
+    q.load(args, b, v, slot, p0, cnt, cg, cn);
+    q.store(args, b, v, p0, cnt, cg, cn);
 }
 
-// Phase B: one CTA per tile of a view; blockIdx.y < N - a: views outside the
-// anchor set (fold the tile's increments); blockIdx.y >= N - a: anchor views
-// (only for an in-place cache update, see phase A).
+// Phase B: one CTA per (tile, group of 4 channels) of a view; blockIdx.y <
+// N - a: views outside the anchor set (fold the tile's increments);
+// blockIdx.y >= N - a: anchor views (only for an in-place cache update, see
+// phase A).
 template <typename T, bool VEC>
-__global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_kernel(const TransportArgs args) {
+__global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_kernel(const TransportArgs args, int n_cg) {
     __shared__ float s_acc[kTileTokens][4];
     __shared__ uint8_t s_n[kTileTokens];
     __shared__ int s_r0[GEOCACHE_MAX_VIEWS], s_cnt[GEOCACHE_MAX_VIEWS];
     const int HW = args.H * args.W;
     const int T_tiles = tiles_per_view_dev(args.H, args.W);
-    const int tile = blockIdx.x, b = blockIdx.z;
+    const int tile = blockIdx.x / n_cg, cg = (blockIdx.x % n_cg) * 4, b = blockIdx.z;
     const int N = args.N, C = args.C, a = args.a;
+    const int cn = C - cg < 4 ? C - cg : 4;
     const int tile0 = tile * kTileTokens;
     const int t = threadIdx.x;
     const int p0 = tile0 + 4 * t;
@@ -1310,18 +1373,15 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
         const int slot = blockIdx.y - (N - a);
         pdl_wait();
         if (cnt <= 0) return;
-        for (int cg = 0; cg < C; cg += 4) {
-            const int cn = C - cg < 4 ? C - cg : 4;
-            QuadRows<T, VEC> q;
-            q.load(args, b, args.anchors[slot], slot, p0, cnt, cg, cn);
-            q.store(args, b, args.anchors[slot], p0, cnt, cg, cn);
-        }
+        QuadRows<T, VEC> q;
+        q.load(args, b, args.anchors[slot], slot, p0, cnt, cg, cn);
+        q.store(args, b, args.anchors[slot], p0, cnt, cg, cn);
         return;
     }
     const int v = nonanchor_view(args, blockIdx.y);
     // streamed rows first (phase A writes none of them), tile offsets next
     QuadRows<T, VEC> q;
-    if (cnt > 0) q.load(args, b, v, -1, p0, cnt, 0, C < 4 ? C : 4);
+    if (cnt > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
     if (t < a) {
         const size_t i = (((size_t)b * N + v) * N + args.anchors[t]) * T_tiles + tile;
         // ranges clamped to the records that exist (an overflow is reported by the build)
@@ -1330,7 +1390,7 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
         s_cnt[t] = record_offset(args.tile_ptr, i + 1, args.max_records) - r0;
     }
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {  // the first channel group's sums, cleared before the wait
+    for (int i = 0; i < 4; ++i) {  // the sums, cleared before the wait
         *reinterpret_cast<float4*>(s_acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
         s_n[4 * t + i] = 0;
     }
@@ -1339,108 +1399,236 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
     int total = 0;
     for (int s2 = 0; s2 < a; ++s2) total += s_cnt[s2];
     if (total == 0) {  // no record in the tile: every token keeps x0(t-1), nothing to fold
-        if (cnt > 0)
-            for (int cg = 0; cg < C; cg += 4) {
-                const int cn = C - cg < 4 ? C - cg : 4;
-                if (cg > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
-                q.store(args, b, v, p0, cnt, cg, cn);
-            }
+        if (cnt > 0) q.store(args, b, v, p0, cnt, cg, cn);
         return;
     }
-    for (int cg = 0; cg < C; cg += 4) {
-        const int cn = C - cg < 4 ? C - cg : 4;
-        if (cg > 0) {
-            if (cnt > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
+    for (int j0 = 0; j0 < total; j0 += kThreads) {
+        const int j = j0 + t;
+        int s_mine = -1, lp = 0;
+        float g[4] = {0.f, 0.f, 0.f, 0.f};
+        if (j < total) {
+            int s2 = 0, jj = j;
+            while (jj >= s_cnt[s2]) jj -= s_cnt[s2++];
+            const int r = s_r0[s2] + jj;
+            lp = (__ldg(&args.records[r].token_mask) & 0x0fffffff) - tile0;
+            const float* w = args.workspace + (size_t)r * C + cg;
+            if (cn == 4 && C % 4 == 0) {
+                const float4 wq = *reinterpret_cast<const float4*>(w);
+                g[0] = wq.x; g[1] = wq.y; g[2] = wq.z; g[3] = wq.w;
+            } else {
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                *reinterpret_cast<float4*>(s_acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
-                s_n[4 * t + i] = 0;
+                for (int c = 0; c < 4; ++c)
+                    if (c < cn) g[c] = w[c];
+            }
+            s_mine = s2;
+        }
+        // combine in anchor order (deterministic): anchor s2 adds in pass s2; the
+        // records are in anchor order, so only the anchors of this round pass
+        int s_lo = 0, c_lo = 0;
+        while (c_lo + s_cnt[s_lo] <= j0) c_lo += s_cnt[s_lo++];
+        const int j_last = (j0 + kThreads < total ? j0 + kThreads : total) - 1;
+        int s_hi = s_lo, c_hi = c_lo;
+        while (c_hi + s_cnt[s_hi] <= j_last) c_hi += s_cnt[s_hi++];
+        for (int s2 = s_lo; s2 <= s_hi; ++s2) {
+            if (s_mine == s2) {
+                float4* dst = reinterpret_cast<float4*>(s_acc[lp]);
+                float4 cur = *dst;
+                cur.x = __fadd_rn(cur.x, g[0]);
+                cur.y = __fadd_rn(cur.y, g[1]);
+                cur.z = __fadd_rn(cur.z, g[2]);
+                cur.w = __fadd_rn(cur.w, g[3]);
+                *dst = cur;
+                s_n[lp] += 1;
             }
             __syncthreads();
         }
-        for (int j0 = 0; j0 < total; j0 += kThreads) {
-            const int j = j0 + t;
-            int s_mine = -1, lp = 0;
-            float g[4] = {0.f, 0.f, 0.f, 0.f};
-            if (j < total) {
-                int s2 = 0, jj = j;
-                while (jj >= s_cnt[s2]) jj -= s_cnt[s2++];
-                const int r = s_r0[s2] + jj;
-                lp = (__ldg(&args.records[r].token_mask) & 0x0fffffff) - tile0;
-                const float* w = args.workspace + (size_t)r * C + cg;
-                if (cn == 4 && C % 4 == 0) {
-                    const float4 wq = *reinterpret_cast<const float4*>(w);
-                    g[0] = wq.x; g[1] = wq.y; g[2] = wq.z; g[3] = wq.w;
-                } else {
-#pragma unroll
-                    for (int c = 0; c < 4; ++c)
-                        if (c < cn) g[c] = w[c];
-                }
-                s_mine = s2;
-            }
-            // combine in anchor order (deterministic): anchor s2 adds in pass s2
-            for (int s2 = 0; s2 < a; ++s2) {
-                if (s_mine == s2) {
-                    float4* dst = reinterpret_cast<float4*>(s_acc[lp]);
-                    float4 cur = *dst;
-                    cur.x = __fadd_rn(cur.x, g[0]);
-                    cur.y = __fadd_rn(cur.y, g[1]);
-                    cur.z = __fadd_rn(cur.z, g[2]);
-                    cur.w = __fadd_rn(cur.w, g[3]);
-                    *dst = cur;
-                    s_n[lp] += 1;
-                }
-                __syncthreads();
-            }
-        }
-        if (cnt > 0) {
-            q.fold(s_acc, s_n, 4 * t, args.update == GEOCACHE_UPDATE_COPY);
-            q.store(args, b, v, p0, cnt, cg, cn);
-        }
-        if (cg + 4 < C) __syncthreads();  // sums are rewritten by the next channel group
+    }
+    if (cnt > 0) {
+        q.fold(s_acc, s_n, 4 * t, args.update == GEOCACHE_UPDATE_COPY);
+        q.store(args, b, v, p0, cnt, cg, cn);
     }
 }
+
+// Phase A by source tile (wide latents): one CTA per (asset, anchor slot,
+// source tile, group of 4 channels).  It stages the anchor's increment
+// x0_new - x0(t-1) (x0_new itself for the value copy) of the tile and of the
+// W + 1 tokens after it in shared memory ([token][4 channels]: every tap of a
+// record whose first kept tap lies in the tile), streams the anchor tile
+// itself (x0(t) and the reconstruction) unless the update is in place, and
+// then applies the tile's group of the source index: for each record whose
+// target view is outside the anchor set, sum_k w_k increment[q_k] in tap
+// order, read from shared memory, into its workspace row.  The scattered
+// per-channel gathers of the record-parallel apply become one coalesced read
+// of the anchor tile.
+template <typename T, int K, bool COPY>
+__global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_src_kernel(const TransportArgs args,
+                                                                                       int n_cg, int stream) {
+    pdl_launch_dependents();
+    extern __shared__ __align__(16) float4 s_d[];  // [kTileTokens + W + 1] tokens x 4 channels
+    const int HW = args.H * args.W, W = args.W;
+    const int N = args.N, C = args.C, a = args.a;
+    const int n_tiles = tiles_per_view_dev(args.H, args.W);
+    long long k = blockIdx.x;
+    const int cg = (int)(k % n_cg) * 4;
+    k /= n_cg;
+    const int st = (int)(k % n_tiles);
+    k /= n_tiles;
+    const int slot = (int)(k % a);
+    const int b = (int)(k / a);
+    const int u = args.anchors[slot];
+    const int cn = C - cg < 4 ? C - cg : 4;
+    const size_t plane = (size_t)HW;
+    const int tile0 = st * kTileTokens;
+    const int span = min(kTileTokens + W + 1, HW - tile0);  // staged tokens
+    const float* xn = args.x0_new + ((size_t)b * a + slot) * C * plane;
+    const float* xp = args.x0_prev + ((size_t)b * N + u) * C * plane;
+    const size_t view_base = ((size_t)b * N + u) * C * plane;
+    const T* xt_p = static_cast<const T*>(args.x_t);
+    T* xn_p = static_cast<T*>(args.x_next);
+    const bool vec_rows = (HW & 3) == 0;
+    for (int q = threadIdx.x; 4 * q < span; q += kThreads) {
+        const int p0 = tile0 + 4 * q;
+        const int cnt = min(4, span - 4 * q);
+        const bool vec = vec_rows && cnt == 4;
+        float dd[4][4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) dd[c][i] = 0.0f;
+            if (c >= cn) continue;
+            float dn[4];
+            f4_load_keep(xn, (size_t)(cg + c) * plane + p0, cnt, vec, dn);
+            if (!COPY) {
+                float pv[4];
+                f4_load_keep(xp, (size_t)(cg + c) * plane + p0, cnt, vec, pv);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) dd[c][i] = __fsub_rn(dn[i], pv[i]);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) dd[c][i] = dn[i];
+            }
+            if (stream && 4 * q < kTileTokens) {  // the anchor tile itself: x0(t) and the reconstruction
+                const size_t e = view_base + (size_t)(cg + c) * plane + p0;
+                Lat4<float>::store(args.x0_out, e, cnt, vec, dn);
+                if (args.coef.enabled) {
+                    float x[4], yv[4], pr[4];
+                    Lat4<T>::load(xt_p, e, cnt, vec, x);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) yv[i] = recon_one(args.coef, x[i], dn[i], pr[i]);
+                    Lat4<T>::store(xn_p, e, cnt, vec, yv);
+                    if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, vec, pr);
+                }
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            if (i < cnt) s_d[4 * q + i] = make_float4(dd[0][i], dd[1][i], dd[2][i], dd[3][i]);
+    }
+    __syncthreads();
+    const size_t grp = ((size_t)b * N + u) * n_tiles + st;  // group ends: see src_index_kernel
+    const int lo = grp ? __ldg(args.src_ptr + grp - 1) : 0, hi = __ldg(args.src_ptr + grp);
+    const int2* src_rec = reinterpret_cast<const int2*>(args.src_rec);
+    for (int e = lo + threadIdx.x; e < hi; e += kThreads) {
+        const int2 ent = __ldg(src_rec + e);
+        if (args.slot_of[ent.y] >= 0) continue;  // target view is an anchor at this step
+        const int4 rec = __ldg(reinterpret_cast<const int4*>(args.records) + ent.x);
+        Taps tp;
+        taps_from_record<K>((int)((uint32_t)rec.x >> 28), rec.y, __int_as_float(rec.z), __int_as_float(rec.w), W, tp);
+        float g[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int kk = 0; kk < K; ++kk) {
+            if (tp.q[kk] < 0) continue;
+            const float4 d = s_d[tp.q[kk] - tile0];
+            g[0] = __fmaf_rn(tp.w[kk], d.x, g[0]);
+            g[1] = __fmaf_rn(tp.w[kk], d.y, g[1]);
+            g[2] = __fmaf_rn(tp.w[kk], d.z, g[2]);
+            g[3] = __fmaf_rn(tp.w[kk], d.w, g[3]);
+        }
+        float* out = args.workspace + (size_t)ent.x * C + cg;
+        if (cn == 4 && C % 4 == 0) {
+            *reinterpret_cast<float4*>(out) = make_float4(g[0], g[1], g[2], g[3]);
+        } else {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (c < cn) out[c] = g[c];
+        }
+    }
+}
+
+// The source-tile apply is used for wide latents (at least kSrcMinChannels
+// channels), where the record-parallel apply's per-channel gathers dominate
+// phase A; with few channels it is slower (it reads the anchors' whole
+// x0(t-1) rows instead of the tapped tokens).
+constexpr int kSrcMinChannels = 8;
+// Record-parallel apply: CTAs per (pair, channel group) sized for about this
+// many records each, from the mean records per ordered view pair.
+constexpr long long kApplyRecords = 384;
 
 template <typename T, int K>
 static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
     const int HW = t.H * t.W;
     const int n_tiles = (HW + kTileTokens - 1) / kTileTokens;
+    const int n_cg = (t.C + 3) / 4;
     const uintptr_t al = (uintptr_t)t.x0_new | (uintptr_t)t.x0_prev | (uintptr_t)t.x0_out | (uintptr_t)t.x_t |
                          (uintptr_t)t.x_next | (uintptr_t)t.pred_out;
     const bool vec = (HW % 4 == 0) && (al % 16 == 0);
     const bool in_place = t.x0_out == t.x0_prev;
-    const int n_slices = (HW + 4095) / 4096;
-    const long long n_apply = t.a < t.N ? (long long)t.B * (t.N - t.a) * t.a * n_slices : 0;
-    const long long n_stream = in_place ? 0 : (long long)t.B * t.a * n_tiles;
-    if (n_apply + n_stream > 0) {
-        if (n_apply + n_stream > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-        const unsigned g = (unsigned)(n_apply + n_stream);
-        const bool copy = t.update == GEOCACHE_UPDATE_COPY;
-        if (vec && !copy)
-            sparse_phase_a_kernel<T, K, true, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
-        else if (vec)
-            sparse_phase_a_kernel<T, K, true, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
-        else if (!copy)
-            sparse_phase_a_kernel<T, K, false, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
+    const bool copy = t.update == GEOCACHE_UPDATE_COPY;
+    // phase A by source tile when the corr has a source index, the latents are
+    // wide and the staged span (tile + W + 1 tokens) fits
+    const bool by_source = t.a < t.N && t.src_ptr && t.src_rec && t.C >= kSrcMinChannels && t.W + 1 <= kTileTokens;
+    bool phase_a = false;
+    if (by_source) {
+        const long long g = (long long)t.B * t.a * n_tiles * n_cg;
+        if (g > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+        const size_t dyn = (size_t)(kTileTokens + t.W + 1) * sizeof(float4);
+        if (!copy)
+            sparse_phase_a_src_kernel<T, K, false><<<(unsigned)g, kThreads, dyn, s>>>(t, n_cg, in_place ? 0 : 1);
         else
-            sparse_phase_a_kernel<T, K, false, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, n_slices);
+            sparse_phase_a_src_kernel<T, K, true><<<(unsigned)g, kThreads, dyn, s>>>(t, n_cg, in_place ? 0 : 1);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
+        phase_a = true;
+    } else {
+        // apply CTAs per (pair, channel group): about kApplyRecords records each
+        const long long pairs = (long long)t.B * t.N * (t.N - 1);
+        const long long per_pair = (t.max_records + pairs - 1) / pairs;
+        long long n_slices = (per_pair + kApplyRecords - 1) / kApplyRecords;
+        n_slices = n_slices < 1 ? 1 : (n_slices > 64 ? 64 : n_slices);
+        const long long n_apply = t.a < t.N ? (long long)t.B * (t.N - t.a) * t.a * n_slices * n_cg : 0;
+        const long long n_stream = in_place ? 0 : (long long)t.B * t.a * n_tiles * n_cg;
+        if (n_apply + n_stream > 0) {
+            if (n_apply + n_stream > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+            const unsigned g = (unsigned)(n_apply + n_stream);
+            const int ns = (int)n_slices;
+            if (vec && !copy)
+                sparse_phase_a_kernel<T, K, true, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, ns, n_cg);
+            else if (vec)
+                sparse_phase_a_kernel<T, K, true, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, ns, n_cg);
+            else if (!copy)
+                sparse_phase_a_kernel<T, K, false, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, ns, n_cg);
+            else
+                sparse_phase_a_kernel<T, K, false, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, ns, n_cg);
+            cudaError_t e = cudaGetLastError();
+            if (e != cudaSuccess) return e;
+            phase_a = true;
+        }
     }
     const int gy = (t.N - t.a) + (in_place ? t.a : 0);
     if (gy > 0) {
+        if ((long long)n_tiles * n_cg > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
         cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3(n_tiles, gy, t.B);
+        cfg.gridDim = dim3((unsigned)(n_tiles * n_cg), gy, t.B);
         cfg.blockDim = dim3(kThreads);
         cfg.dynamicSmemBytes = 0;
         cfg.stream = s;
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-        attr[0].val.programmaticStreamSerializationAllowed = n_apply + n_stream > 0 ? 1 : 0;
+        attr[0].val.programmaticStreamSerializationAllowed = phase_a ? 1 : 0;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        cudaError_t e = vec ? cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true>, t)
-                            : cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false>, t);
+        cudaError_t e = vec ? cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true>, t, n_cg)
+                            : cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false>, t, n_cg);
         if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();

@@ -48,7 +48,8 @@ class Corr(ctypes.Structure):
                 ("pos", ctypes.c_void_p), ("valid", ctypes.c_void_p), ("cams", ctypes.c_void_p),
                 ("tau", ctypes.c_void_p), ("idx", ctypes.c_void_p), ("w", ctypes.c_void_p),
                 ("keep", ctypes.c_void_p), ("tile_ptr", ctypes.c_void_p), ("records", ctypes.c_void_p),
-                ("max_records", ctypes.c_int64), ("mode", ctypes.c_int)]
+                ("max_records", ctypes.c_int64), ("mode", ctypes.c_int),
+                ("src_ptr", ctypes.c_void_p), ("src_rec", ctypes.c_void_p)]
 
 
 class Recon(ctypes.Structure):
@@ -204,15 +205,16 @@ def tiles_per_view(H: int, W: int) -> int:
 
 
 def make_corr(pos, valid, cams, tau, idx=None, w=None, K=4, tol_frac=0.01, mode=None, keep=None,
-              tile_ptr=None, records=None) -> CorrHandle:
+              tile_ptr=None, records=None, src_ptr=None, src_rec=None) -> CorrHandle:
     """Describe a batch's geometry (and optional tables, keep masks and sparse
     form) for the C ABI.  records is an int32 tensor [R, 4] (16-byte tap
-    records).  The default mode is SPARSE when records are given, else MASK
+    records); src_ptr [B*N*T + 1] and src_rec [R, 2] int32 hold the optional
+    source index.  The default mode is SPARSE when records are given, else MASK
     when keep masks are given, else TABLE when tables are given, else GEOMETRY."""
     B, N, H, W = valid.shape
     n = B * N * H * W
     refs = {"pos": pos, "valid": valid, "cams": cams, "tau": tau, "idx": idx, "w": w, "keep": keep,
-            "tile_ptr": tile_ptr, "records": records}
+            "tile_ptr": tile_ptr, "records": records, "src_ptr": src_ptr, "src_rec": src_rec}
     if mode is None:
         mode = (CORR_SPARSE if records is not None else CORR_MASK if keep is not None
                 else CORR_TABLE if idx is not None else CORR_GEOMETRY)
@@ -224,7 +226,9 @@ def make_corr(pos, valid, cams, tau, idx=None, w=None, K=4, tol_frac=0.01, mode=
              _dev(idx, torch.int32, n * N * K, "idx"), _dev(w, torch.float32, n * N * K, "w"),
              _dev(keep, torch.uint8, n * N, "keep"),
              _dev(tile_ptr, torch.int32, B * N * N * tiles_per_view(H, W) + 1, "tile_ptr"),
-             _dev(records, torch.int32, None, "records"), 0 if records is None else records.shape[0], mode)
+             _dev(records, torch.int32, None, "records"), 0 if records is None else records.shape[0], mode,
+             _dev(src_ptr, torch.int32, B * N * tiles_per_view(H, W) + 1, "src_ptr"),
+             _dev(src_rec, torch.int32, None if records is None else 2 * records.shape[0], "src_rec"))
     return CorrHandle(c, refs)
 
 
@@ -235,10 +239,13 @@ def record_count(corr: CorrHandle, stream=None) -> int:
     return int(n.value)
 
 
-def build_sparse_corr(pos, valid, cams, K=4, tol_frac=0.01, tables=False, stream=None) -> CorrHandle:
+def build_sparse_corr(pos, valid, cams, K=4, tol_frac=0.01, tables=False, stream=None,
+                      source_index=False) -> CorrHandle:
     """Allocate and build the full correspondence state of a batch: tau, keep
-    masks, the sparse form (count, then records) and optionally the tables.
-    Allocation happens here, once per batch of assets, never per step."""
+    masks, the sparse form (count, then records), optionally the tables and
+    the source index (worth building for latents of 8 or more channels, whose
+    steps then apply the records per source tile).  Allocation happens here,
+    once per batch of assets, never per step."""
     B, N, H, W = valid.shape
     dev = pos.device
     tau = torch.zeros(B, dtype=torch.float32, device=dev)
@@ -252,8 +259,12 @@ def build_sparse_corr(pos, valid, cams, K=4, tol_frac=0.01, tables=False, stream
     if tables:
         idx = torch.empty((B, N, N, H, W, K), dtype=torch.int32, device=dev)
         w = torch.empty((B, N, N, H, W, K), dtype=torch.float32, device=dev)
+    src_ptr = src_rec = None
+    if source_index:
+        src_ptr = torch.empty(B * N * tiles_per_view(H, W) + 1, dtype=torch.int32, device=dev)
+        src_rec = torch.empty((records.shape[0], 2), dtype=torch.int32, device=dev)
     corr = make_corr(pos, valid, cams, tau, idx=idx, w=w, K=K, tol_frac=tol_frac, keep=keep, tile_ptr=tile_ptr,
-                     records=records, mode=CORR_SPARSE)
+                     records=records, mode=CORR_SPARSE, src_ptr=src_ptr, src_rec=src_rec)
     return build_corr(corr, stream)
 
 
@@ -334,9 +345,11 @@ def permute_records(corr: CorrHandle, perm, out=None, stream=None) -> CorrHandle
     refs = dict(corr._keep)
     refs["records"] = out
     refs["perm"] = perm
+    refs["src_ptr"] = refs["src_rec"] = None
     c2 = Corr.from_buffer_copy(c)
     c2.records = out.data_ptr()
     c2.mode = CORR_SPARSE
+    c2.src_ptr = c2.src_rec = None  # the source index belongs to the unpermuted records
     return CorrHandle(c2, refs)
 
 

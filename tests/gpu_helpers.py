@@ -128,7 +128,7 @@ class DeviceGeometry:
     (optionally) the idx/w tables, built by geocache_build_corr.  `corr`
     uses the keep masks (the fast path); corr_for(mode) gives the others."""
 
-    def __init__(self, w, K=4, tables=True, dev="cuda"):
+    def __init__(self, w, K=4, tables=True, dev="cuda", source_index=True):
         from paper_2608_13255_gb300 import geocache as gc
         self.gc = gc
         self.w = w
@@ -149,18 +149,26 @@ class DeviceGeometry:
                           tile_ptr=self.tile_ptr, mode=gc.CORR_MASK)
         self.n_records = gc.record_count(c0)
         self.records = torch.empty((max(self.n_records, 1), 4), dtype=torch.int32, device=dev)
+        # source index of the records (used by sparse steps with C >= 8)
+        self.src_ptr = self.src_rec = None
+        if source_index:
+            self.src_ptr = torch.empty(w.B * w.N * gc.tiles_per_view(w.H, w.W) + 1, dtype=torch.int32, device=dev)
+            self.src_rec = torch.empty((self.records.shape[0], 2), dtype=torch.int32, device=dev)
         self.corr = gc.make_corr(self.pos, self.valid, self.cams, self.tau, self.idx, self.wt, K=K,
                                  tol_frac=w.tol_frac, keep=self.keep, tile_ptr=self.tile_ptr, records=self.records,
-                                 mode=gc.CORR_SPARSE)
+                                 mode=gc.CORR_SPARSE, src_ptr=self.src_ptr, src_rec=self.src_rec)
         gc.build_corr(self.corr)
 
     def corr_for(self, mode):
+        """The corr in another mode; 'sparse_plain' is the sparse form without
+        its source index (the record-parallel apply at any C)."""
         gc = self.gc
         m = {"mask": gc.CORR_MASK, "geometry": gc.CORR_GEOMETRY, "table": gc.CORR_TABLE,
-             "sparse": gc.CORR_SPARSE}[mode]
+             "sparse": gc.CORR_SPARSE, "sparse_plain": gc.CORR_SPARSE}[mode]
+        src = mode == "sparse"
         return gc.make_corr(self.pos, self.valid, self.cams, self.tau, self.idx, self.wt, K=self.K,
                             tol_frac=self.w.tol_frac, keep=self.keep, tile_ptr=self.tile_ptr, records=self.records,
-                            mode=m)
+                            mode=m, src_ptr=self.src_ptr if src else None, src_rec=self.src_rec if src else None)
 
     def workspace(self, C):
         return torch.empty(max(self.corr.workspace_floats(C), 4), dtype=torch.float32, device=self.pos.device)

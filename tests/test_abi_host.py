@@ -35,7 +35,7 @@ def test_exports_every_declared_symbol(gc):
     L = gc.load()
     for n in names:
         assert hasattr(L, n), n
-    assert gc.abi_version() == 1
+    assert gc.abi_version() == 2
 
 
 SCHEDS = [

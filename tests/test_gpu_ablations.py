@@ -59,14 +59,14 @@ def test_value_copy_parity(gc, workloads, name):
     params = synth.recon_params(w, 2)
     tau = oracle.tau(w.pos, w.valid, w.tol_frac)
     outs = {}
-    for mode in ("sparse", "mask", "geometry", "table"):
+    for mode in ("sparse", "sparse_plain", "mask", "geometry", "table"):
         (x0_prev, x0_new, xt64), got, d_xn = _gpu_step(gc, w, g, g.corr_for(mode), anchors, params, "copy")
         ref_x0, ref_xn, _ = oracle.transport_step(anchors, x0_new, x0_prev, K=w.K,
                                                   geom=(w.pos, w.valid, w.cams, tau), x_t=xt64,
                                                   recon=recon_kw(params, None), update="copy")
         _check(w, got, d_xn, ref_x0, ref_xn)
         outs[mode] = got
-    for mode in ("mask", "geometry", "table"):  # the modes give the same taps, weights and results
+    for mode in ("sparse_plain", "mask", "geometry", "table"):  # the same taps, weights and results
         np.testing.assert_array_equal(outs[mode], outs["sparse"])
     # the copy really differs from the delta transport on covered targets
     _, got_delta, _ = _gpu_step(gc, w, g, g.corr, anchors, params, "delta")

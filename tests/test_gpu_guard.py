@@ -72,18 +72,23 @@ def _geometry(gc, w, K=4, skew=0, records_frac=1.0):
         "records": Guarded((cap, 4), torch.int32, 0),  # the ABI requires 16-byte aligned records
         "idx": Guarded((w.B, w.N, w.N, w.H, w.W, K), torch.int32, 0 if K == 4 else skew),
         "w": Guarded((w.B, w.N, w.N, w.H, w.W, K), torch.float32, 0 if K == 4 else skew),
+        "src_ptr": Guarded((w.B * w.N * T + 1,), torch.int32, skew),
+        "src_rec": Guarded((cap, 2), torch.int32, 0),  # 8-byte aligned
     }
     corr = gc.make_corr(pos, valid, cams, g["tau"].t, g["idx"].t, g["w"].t, K=K, keep=g["keep"].t,
-                        tile_ptr=g["tile_ptr"].t, records=g["records"].t, mode=gc.CORR_SPARSE)
+                        tile_ptr=g["tile_ptr"].t, records=g["records"].t, mode=gc.CORR_SPARSE,
+                        src_ptr=g["src_ptr"].t, src_rec=g["src_rec"].t)
     gc.build_corr(corr)
     torch.cuda.synchronize()
     return corr, g, R, cap, (pos, valid, cams)
 
 
-@pytest.mark.parametrize("case", ["ragged_c5", "misaligned", "c3_k1"])
+@pytest.mark.parametrize("case", ["ragged_c5", "ragged_c18", "misaligned", "c3_k1"])
 def test_transport_writes_only_its_outputs(gc, case):
     if case == "ragged_c5":  # 37 x 53 tokens: H*W = 1961, two tiles, a ragged quad; C = 5
         w, C, skew, K = synth.make_workload("batch128", B=2, H=37, W=53), 5, 0, 4
+    elif case == "ragged_c18":  # the same with C = 18: the source-tile apply, a partial last channel group
+        w, C, skew, K = synth.make_workload("batch128", B=2, H=37, W=53), 18, 0, 4
     elif case == "misaligned":  # 64 x 64 tokens, every buffer 4 bytes off a 16-byte boundary
         w, C, skew, K = synth.make_workload("hunyuan64"), 4, 4, 4
     else:
@@ -100,8 +105,11 @@ def test_transport_writes_only_its_outputs(gc, case):
     pred_kind = "v" if p["sampler"] == "ddim" else "velocity"
     for mode in ("sparse", "mask", "table", "geometry"):
         m = {"sparse": gc.CORR_SPARSE, "mask": gc.CORR_MASK, "table": gc.CORR_TABLE, "geometry": gc.CORR_GEOMETRY}[mode]
+        src = mode == "sparse"
         c2 = gc.make_corr(corr._keep["pos"], corr._keep["valid"], corr._keep["cams"], corr.tau, corr.idx, corr.w, K=K,
-                          keep=corr.keep, tile_ptr=corr._keep["tile_ptr"], records=corr._keep["records"], mode=m)
+                          keep=corr.keep, tile_ptr=corr._keep["tile_ptr"], records=corr._keep["records"], mode=m,
+                          src_ptr=corr._keep["src_ptr"] if src else None,
+                          src_rec=corr._keep["src_rec"] if src else None)
         out = Guarded(shp, torch.float32, skew)
         xn = Guarded(shp, lat, skew)
         pred = Guarded(shp, torch.float32, skew)

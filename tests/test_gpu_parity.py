@@ -452,3 +452,88 @@ def test_identity_camera_reproduces_anchor_delta(gc, workloads, scene, K):
     err = np.abs((got.astype(np.float64) - prev)[:, fg] - d0[:, fg].astype(np.float64))
     assert err.max() <= 1e-5, err.max()
     print("%s K=%d: %d foreground tokens, max |x0(t) - x0(t-1) - delta| %.3g" % (scene, K, fg.sum(), err.max()))
+
+
+def _source_groups(g, w):
+    """Expected source index from the records: for every record r of pair
+    (b, v, u), its group (b, u, tile of its first kept tap) and target v."""
+    T = g.gc.tiles_per_view(w.H, w.W)
+    rec = g.records.cpu().numpy()[: g.n_records].astype(np.int64)
+    tp = g.tile_ptr.cpu().numpy().astype(np.int64)
+    pair = np.repeat(np.arange(w.B * w.N * w.N), tp[T::T] - tp[:-1:T])  # (b, v, u) of each record
+    b, v, u = pair // (w.N * w.N), (pair // w.N) % w.N, pair % w.N
+    mask, q_tl = (rec[:, 0] >> 28) & 15, rec[:, 1]
+    low = np.array([0, 0, 1, 0, 2, 0, 1, 0, 3, 0, 1, 0, 2, 0, 1, 0])[mask]  # lowest kept tap
+    q = q_tl + (low & 1) + (low >> 1) * w.W if w.K == 4 else q_tl
+    return (b * w.N + u) * T + q // 1024, v
+
+
+@pytest.mark.parametrize("name", ["ring12_128", "solids96"])
+def test_source_index_groups_every_record_once(gc, workloads, name):
+    # the source index (records grouped by the tile of their first kept tap in
+    # the source view) holds each record exactly once, in the right group,
+    # with its target view
+    w = workloads(name)
+    g = DeviceGeometry(w, K=w.K, tables=False)
+    torch.cuda.synchronize()
+    grp, v = _source_groups(g, w)
+    ends = g.src_ptr.cpu().numpy().astype(np.int64)
+    starts = np.concatenate([[0], ends[:-2]])
+    ent = g.src_rec.cpu().numpy()[: g.n_records]
+    assert ends[-2] == ends[-1] == g.n_records
+    np.testing.assert_array_equal(ends[:-1] - starts, np.bincount(grp, minlength=len(ends) - 1))
+    got_grp = np.repeat(np.arange(len(ends) - 1), ends[:-1] - starts)
+    order = np.argsort(ent[:, 0], kind="stable")
+    np.testing.assert_array_equal(np.sort(ent[:, 0]), np.arange(g.n_records))  # every record once
+    np.testing.assert_array_equal(got_grp[order], grp)
+    np.testing.assert_array_equal(ent[order, 1], v)
+
+
+@pytest.mark.parametrize("C,update,inplace", [(16, "delta", False), (16, "delta", True), (20, "copy", False),
+                                              (33, "delta", False), (8, "copy", True)])
+def test_source_tile_apply_equals_record_parallel_apply(gc, workloads, C, update, inplace):
+    # wide latents (C >= 8) apply the records per source tile when the corr
+    # has a source index: bitwise the results of the record-parallel apply, and
+    # the oracle's
+    w = workloads("ring12_128") if C == 16 else workloads("solids96")
+    w = synth.Workload(**{**w.__dict__, "C": C})
+    g = DeviceGeometry(w, K=w.K, tables=False)
+    anchors = oracle.rotate_anchors(w.N, w.a, 1)
+    params = synth.recon_params(w, 8)
+    outs = {}
+    for mode in ("sparse", "sparse_plain"):
+        x0_prev, x0_new, xt32 = step_inputs(w, 3, anchors)
+        xt64, xt = latent_values(xt32, w)
+        d_prev, d_new, d_xt = torch.from_numpy(x0_prev).cuda(), torch.from_numpy(x0_new).cuda(), xt.cuda()
+        d_out = d_prev if inplace else torch.empty_like(d_prev)
+        d_xn = d_xt if inplace else torch.empty_like(d_xt)
+        r = gc.make_recon(params["sampler"], a_t=params.get("a_t", 0), a_prev=params.get("a_prev", 0),
+                          sigma=params.get("sigma", 0), sigma_next=params.get("sigma_next", 0))
+        gc.transport_step(g.corr_for(mode), anchors, C, d_new, d_prev, d_out, d_xt, d_xn, r,
+                          workspace=g.workspace(C), update=update)
+        torch.cuda.synchronize()
+        gc.device_status()
+        outs[mode] = (d_out.cpu().numpy(), d_xn.cpu().view(torch.int16).numpy())
+    np.testing.assert_array_equal(outs["sparse"][0], outs["sparse_plain"][0])
+    np.testing.assert_array_equal(outs["sparse"][1], outs["sparse_plain"][1])
+    tau = oracle.tau(w.pos, w.valid, w.tol_frac)
+    ref_x0, ref_xn, _ = oracle.transport_step(anchors, x0_new, x0_prev, K=w.K, geom=(w.pos, w.valid, w.cams, tau),
+                                              x_t=xt64, recon=recon_kw(params), update=update)
+    assert_f32_close(outs["sparse"][0], ref_x0, what="x0")
+    assert_bf16_close(outs["sparse"][1].view(np.uint16), ref_xn, what="x_next")
+
+
+def test_wide_views_fall_back_to_the_record_parallel_apply(gc):
+    # W + 1 > 1024 tokens: the staged span of a source tile would not fit, so a
+    # step with a source index applies the records record-parallel; results
+    # equal the oracle's
+    H, W = 16, 1040
+    w = synth.make_workload("solids96", H=H, W=W)
+    cams = np.stack([synth.look_at_camera(az, el, W, W) for az, el in synth.hunyuan_layout()])
+    cams[:, 15] = H / 2.0  # a 16-row strip through the middle of a square camera's image
+    pos, valid = synth.render_asset(synth.unit_sphere(), cams, H, W)
+    w = synth.Workload(**{**w.__dict__, "C": 8, "cams": cams[None].astype(np.float32), "pos": pos[None],
+                          "valid": valid[None]})
+    g = DeviceGeometry(w, K=4, tables=False)
+    assert g.n_records > 100
+    _run_step(gc, w, g, [0, 2, 4], synth.recon_params(w, 5))
