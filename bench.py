@@ -442,15 +442,20 @@ class Trajectory:
             wt = torch.empty(shp, dtype=torch.float32, device=dev)
         if corr_mode in ("mask", "sparse"):
             keep = torch.empty((w.B, w.N, w.N, w.H, w.W), dtype=torch.uint8, device=dev)
+        src_ptr = src_rec = None
         if corr_mode == "sparse":
             tile_ptr = torch.empty(w.B * w.N * w.N * gc.tiles_per_view(w.H, w.W) + 1, dtype=torch.int32, device=dev)
             c0 = gc.make_corr(self.pos, self.valid, self.cams, self.tau, K=w.K, tol_frac=w.tol_frac, keep=keep,
                               tile_ptr=tile_ptr, mode=gc.CORR_MASK)
             records = torch.empty((max(gc.record_count(c0), 1), 4), dtype=torch.int32, device=dev)
+            if w.C >= 8:  # wide latents: the source index for the source-tile apply
+                src_ptr = torch.empty(w.B * w.N * gc.tiles_per_view(w.H, w.W) + 1, dtype=torch.int32, device=dev)
+                src_rec = torch.empty((records.shape[0], 2), dtype=torch.int32, device=dev)
         mode = {"mask": gc.CORR_MASK, "table": gc.CORR_TABLE, "geometry": gc.CORR_GEOMETRY,
                 "sparse": gc.CORR_SPARSE}[corr_mode]
         self.corr = gc.make_corr(self.pos, self.valid, self.cams, self.tau, idx, wt, K=w.K, tol_frac=w.tol_frac,
-                                 mode=mode, keep=keep, tile_ptr=tile_ptr, records=records)
+                                 mode=mode, keep=keep, tile_ptr=tile_ptr, records=records, src_ptr=src_ptr,
+                                 src_rec=src_rec)
         nws = self.corr.workspace_floats(w.C)
         self.workspace = torch.empty(max(nws, 4), dtype=torch.float32, device=dev) if nws else None
         xT, x0 = synth.initial_latents(w)
@@ -491,7 +496,9 @@ class Trajectory:
         gc.build_corr(self.corr)
         launches += 1 + (1 if (self.corr.idx is not None or self.corr.keep is not None) else 0)
         if self.corr.c.mode == gc.CORR_SPARSE:
-            launches += 3  # tile counts, their scan, the records
+            launches += 2  # the tile offsets' scan, the records
+            if self.corr.c.src_ptr:
+                launches += 3  # the source index: counts, their scan, the scatter
         cache = None
         for t in range(w.S):
             timed = events is not None and t in self.anchor_x0
@@ -981,7 +988,7 @@ def main():
                      "kernel": "sparse_phase_a_kernel + sparse_phase_b_kernel (one cached step)",
                      "alg_bytes_per_launch": alg,
                      "avg_launch_us": 1e3 * k_avg_ms, "launches": len(kernel_ms),
-                     "timed_by": "events around each cached step's graph replay",
+                     "timed_by": "events around each cached step's graph replay (launch included)",
                      "frac_of_8TBs": achieved / 8000.0},
         "gpu_launches": launches,
         "pack_anchors": pack,

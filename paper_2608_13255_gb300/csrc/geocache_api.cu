@@ -328,8 +328,10 @@ int geocache_transport_step_update(const geocache_corr* c, geocache_update updat
     t.x0_new = x0_anchor_new; t.x0_prev = x0_prev; t.x0_out = x0_out;
     t.x_t = x_t; t.x_next = x_next; t.pred_out = recon ? recon->pred_out : nullptr;
     t.coef = coef;
-    for (int v = 0; v < GEOCACHE_MAX_VIEWS; ++v) { t.slot_of[v] = -1; t.anchors[v] = -1; }
+    for (int v = 0; v < GEOCACHE_MAX_VIEWS; ++v) { t.slot_of[v] = -1; t.anchors[v] = -1; t.others[v] = -1; }
     for (int s = 0; s < a; ++s) { t.anchors[s] = anchors[s]; t.slot_of[anchors[s]] = s; }
+    for (int v = 0, k = 0; v < c->N; ++v)
+        if (t.slot_of[v] < 0) t.others[k++] = v;
     cudaStream_t s = (cudaStream_t)stream;
     t.c0 = 0;
     t.cn = C;

@@ -50,6 +50,7 @@ struct TransportArgs {
     ReconCoef coef;
     int32_t anchors[GEOCACHE_MAX_VIEWS];
     int32_t slot_of[GEOCACHE_MAX_VIEWS];   // slot in `anchors`, -1 for non-anchors
+    int32_t others[GEOCACHE_MAX_VIEWS];    // the views outside the anchor set, ascending
 };
 
 struct RowAnchors {

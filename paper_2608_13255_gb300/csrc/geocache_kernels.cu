@@ -1189,16 +1189,32 @@ struct QuadRows {
         }
     }
 
-    // add the folded increments of the tile (mean over covering anchors)
-    __device__ __forceinline__ void fold(const float (*s_acc)[4], const uint8_t* s_n, int lp0, bool copy) {
+    // add the folded increments of the quad's tokens (the mean over their
+    // covering anchors, Eq. 1 with the aggregation of Sec. 3.2): n4 holds the
+    // four tokens' anchor counts, one byte each; g / n is a multiplication
+    // for n a power of two (exact) and a division otherwise
+    template <bool COPY>
+    __device__ __forceinline__ void fold4(const float (*s_acc)[4], uint32_t n4, int lp0) {
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            const int n = s_n[lp0 + i];
+            const int n = (int)((n4 >> (8 * i)) & 0xffu);
             if (!n) continue;
             const float4 gq = *reinterpret_cast<const float4*>(s_acc[lp0 + i]);
             const float gg[4] = {gq.x, gq.y, gq.z, gq.w};
+            float m[4];
+            if (n == 1) {
 #pragma unroll
-            for (int c = 0; c < 4; ++c) x0[c][i] = fold_one(copy, x0[c][i], gg[c], n);
+                for (int c = 0; c < 4; ++c) m[c] = gg[c];
+            } else if ((n & (n - 1)) == 0) {
+                const float rn = __frcp_rn((float)n);
+#pragma unroll
+                for (int c = 0; c < 4; ++c) m[c] = __fmul_rn(gg[c], rn);
+            } else {
+#pragma unroll
+                for (int c = 0; c < 4; ++c) m[c] = __fdiv_rn(gg[c], (float)n);
+            }
+#pragma unroll
+            for (int c = 0; c < 4; ++c) x0[c][i] = COPY ? m[c] : __fadd_rn(x0[c][i], m[c]);
         }
     }
 
@@ -1230,12 +1246,6 @@ struct QuadRows {
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
-// the v-th view outside the anchor set
-__device__ __forceinline__ int nonanchor_view(const TransportArgs& args, int vi) {
-    for (int x = 0, r = 0; x < args.N; ++x)
-        if (args.slot_of[x] < 0 && r++ == vi) return x;
-    return -1;
-}
 
 // Tile offset i of the sparse form clamped to the records that exist, [0,
 // cap]: a build whose records overflowed the capacity or the int32 offsets
@@ -1257,7 +1267,7 @@ __device__ __forceinline__ void apply_records(const TransportArgs& args, int pai
     const int s2 = pair_id % a;
     const int vi = (pair_id / a) % (N - a);
     const int b = pair_id / (a * (N - a));
-    const int v = nonanchor_view(args, vi);
+    const int v = args.others[vi];
     const int u = args.anchors[s2];
     const size_t pair = ((size_t)b * N + v) * N + u;
     const long long cap = args.max_records;
@@ -1355,10 +1365,10 @@ __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_ker
 // N - a: views outside the anchor set (fold the tile's increments);
 // blockIdx.y >= N - a: anchor views (only for an in-place cache update, see
 // phase A).
-template <typename T, bool VEC>
+template <typename T, bool VEC, bool COPY>
 __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_kernel(const TransportArgs args, int n_cg) {
     __shared__ float s_acc[kTileTokens][4];
-    __shared__ uint8_t s_n[kTileTokens];
+    __shared__ __align__(4) uint8_t s_n[kTileTokens];
     __shared__ int s_r0[GEOCACHE_MAX_VIEWS], s_cnt[GEOCACHE_MAX_VIEWS];
     const int HW = args.H * args.W;
     const int T_tiles = tiles_per_view_dev(args.H, args.W);
@@ -1378,7 +1388,7 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
         q.store(args, b, args.anchors[slot], p0, cnt, cg, cn);
         return;
     }
-    const int v = nonanchor_view(args, blockIdx.y);
+    const int v = args.others[blockIdx.y];
     // streamed rows first (phase A writes none of them), tile offsets next
     QuadRows<T, VEC> q;
     if (cnt > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
@@ -1444,7 +1454,8 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
         }
     }
     if (cnt > 0) {
-        q.fold(s_acc, s_n, 4 * t, args.update == GEOCACHE_UPDATE_COPY);
+        const uint32_t n4 = *reinterpret_cast<const uint32_t*>(s_n + 4 * t);
+        if (n4) q.template fold4<COPY>(s_acc, n4, 4 * t);
         q.store(args, b, v, p0, cnt, cg, cn);
     }
 }
@@ -1627,8 +1638,11 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
         attr[0].val.programmaticStreamSerializationAllowed = phase_a ? 1 : 0;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        cudaError_t e = vec ? cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true>, t, n_cg)
-                            : cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false>, t, n_cg);
+        cudaError_t e;
+        if (vec && !copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, false>, t, n_cg);
+        else if (vec) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, true>, t, n_cg);
+        else if (!copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, false>, t, n_cg);
+        else e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, true>, t, n_cg);
         if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();
