@@ -1404,10 +1404,19 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
         *reinterpret_cast<float4*>(s_acc[4 * t + i]) = make_float4(0.f, 0.f, 0.f, 0.f);
         s_n[4 * t + i] = 0;
     }
-    pdl_wait();  // phase A's workspace writes are complete and visible
     __syncthreads();
     int total = 0;
     for (int s2 = 0; s2 < a; ++s2) total += s_cnt[s2];
+    // a tile without records keeps x0(t-1) and reads and writes nothing phase A
+    // touches (rows of views outside the anchor set), so it is stored without
+    // waiting for phase A; the first CTA always waits, so that this grid
+    // completes only after phase A
+    const bool first = blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0;
+    if (total == 0 && !first) {
+        if (cnt > 0) q.store(args, b, v, p0, cnt, cg, cn);
+        return;
+    }
+    pdl_wait();  // phase A's workspace writes are complete and visible
     if (total == 0) {  // no record in the tile: every token keeps x0(t-1), nothing to fold
         if (cnt > 0) q.store(args, b, v, p0, cnt, cg, cn);
         return;
@@ -1539,29 +1548,42 @@ __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_src
     const size_t grp = ((size_t)b * N + u) * n_tiles + st;  // group ends: see src_index_kernel
     const int lo = grp ? __ldg(args.src_ptr + grp - 1) : 0, hi = __ldg(args.src_ptr + grp);
     const int2* src_rec = reinterpret_cast<const int2*>(args.src_rec);
-    for (int e = lo + threadIdx.x; e < hi; e += kThreads) {
-        const int2 ent = __ldg(src_rec + e);
-        if (args.slot_of[ent.y] >= 0) continue;  // target view is an anchor at this step
-        const int4 rec = __ldg(reinterpret_cast<const int4*>(args.records) + ent.x);
-        Taps tp;
-        taps_from_record<K>((int)((uint32_t)rec.x >> 28), rec.y, __int_as_float(rec.z), __int_as_float(rec.w), W, tp);
-        float g[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int e0 = lo + threadIdx.x; e0 < hi; e0 += 2 * kThreads) {
+        // two entries per thread, their loads in flight together
+        int2 ent[2];
+        int4 rec[2];
 #pragma unroll
-        for (int kk = 0; kk < K; ++kk) {
-            if (tp.q[kk] < 0) continue;
-            const float4 d = s_d[tp.q[kk] - tile0];
-            g[0] = __fmaf_rn(tp.w[kk], d.x, g[0]);
-            g[1] = __fmaf_rn(tp.w[kk], d.y, g[1]);
-            g[2] = __fmaf_rn(tp.w[kk], d.z, g[2]);
-            g[3] = __fmaf_rn(tp.w[kk], d.w, g[3]);
+        for (int m = 0; m < 2; ++m) {
+            const int e = e0 + m * kThreads;
+            ent[m] = e < hi ? __ldg(src_rec + e) : make_int2(-1, 0);
+            if (ent[m].x >= 0 && args.slot_of[ent[m].y] >= 0) ent[m].x = -1;  // target view is an anchor
+            rec[m] = ent[m].x >= 0 ? __ldg(reinterpret_cast<const int4*>(args.records) + ent[m].x)
+                                   : make_int4(0, 0, 0, 0);
         }
-        float* out = args.workspace + (size_t)ent.x * C + cg;
-        if (cn == 4 && C % 4 == 0) {
-            *reinterpret_cast<float4*>(out) = make_float4(g[0], g[1], g[2], g[3]);
-        } else {
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
-                if (c < cn) out[c] = g[c];
+        for (int m = 0; m < 2; ++m) {
+            if (ent[m].x < 0) continue;
+            Taps tp;
+            taps_from_record<K>((int)((uint32_t)rec[m].x >> 28), rec[m].y, __int_as_float(rec[m].z),
+                                __int_as_float(rec[m].w), W, tp);
+            float g[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int kk = 0; kk < K; ++kk) {
+                if (tp.q[kk] < 0) continue;
+                const float4 d = s_d[tp.q[kk] - tile0];
+                g[0] = __fmaf_rn(tp.w[kk], d.x, g[0]);
+                g[1] = __fmaf_rn(tp.w[kk], d.y, g[1]);
+                g[2] = __fmaf_rn(tp.w[kk], d.z, g[2]);
+                g[3] = __fmaf_rn(tp.w[kk], d.w, g[3]);
+            }
+            float* out = args.workspace + (size_t)ent[m].x * C + cg;
+            if (cn == 4 && C % 4 == 0) {
+                *reinterpret_cast<float4*>(out) = make_float4(g[0], g[1], g[2], g[3]);
+            } else {
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+                    if (c < cn) out[c] = g[c];
+            }
         }
     }
 }
