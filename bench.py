@@ -248,7 +248,7 @@ def time_cached_steps(w, B, dev, reps=24, seed=3):
     from paper_2608_13255_gb300 import synth
     wb = synth.replicate_assets(w, B)
     pos, valid, cams = (torch.from_numpy(a).to(dev) for a in (wb.pos, wb.valid, wb.cams))
-    corr = gc.build_sparse_corr(pos, valid, cams, K=wb.K, tol_frac=wb.tol_frac, source_index=wb.C >= 8)
+    corr = gc.build_sparse_corr(pos, valid, cams, K=wb.K, tol_frac=wb.tol_frac)
     wsp = torch.empty(max(corr.workspace_floats(wb.C), 4), dtype=torch.float32, device=dev)
     cached = [t for t in range(wb.S) if not gc.rotate_anchors(wb.N, wb.a, t, wb.S, wb.schedule)[1]]
     sets = []
@@ -448,9 +448,6 @@ class Trajectory:
             c0 = gc.make_corr(self.pos, self.valid, self.cams, self.tau, K=w.K, tol_frac=w.tol_frac, keep=keep,
                               tile_ptr=tile_ptr, mode=gc.CORR_MASK)
             records = torch.empty((max(gc.record_count(c0), 1), 4), dtype=torch.int32, device=dev)
-            if w.C >= 8:  # wide latents: the source index for the source-tile apply
-                src_ptr = torch.empty(w.B * w.N * gc.tiles_per_view(w.H, w.W) + 1, dtype=torch.int32, device=dev)
-                src_rec = torch.empty((records.shape[0], 2), dtype=torch.int32, device=dev)
         mode = {"mask": gc.CORR_MASK, "table": gc.CORR_TABLE, "geometry": gc.CORR_GEOMETRY,
                 "sparse": gc.CORR_SPARSE}[corr_mode]
         self.corr = gc.make_corr(self.pos, self.valid, self.cams, self.tau, idx, wt, K=w.K, tol_frac=w.tol_frac,

@@ -65,8 +65,11 @@ typedef enum {
     GEOCACHE_CORR_TABLE = 1,    /* read idx/w written by geocache_build_corr (or supplied by the caller) */
     GEOCACHE_CORR_MASK = 2,     /* read the 1-byte keep masks written by geocache_build_corr; recompute
                                    the projection and weights only where a tap is kept */
-    GEOCACHE_CORR_SPARSE = 3    /* read the sparse tap records written by geocache_build_corr and apply
-                                   them record-parallel into a workspace (fastest) */
+    GEOCACHE_CORR_SPARSE = 3    /* read the sparse tap records written by geocache_build_corr (fastest):
+                                   C < 8, or a workspace without room for the increment plane: the
+                                   records are applied record-parallel (or per source tile with a
+                                   source index) into workspace rows; C >= 8 with room: the anchors'
+                                   increments are written as a plane and gathered per record */
 } geocache_corr_mode;
 
 /* Update rule of the views outside the anchor set at a cached step. */
@@ -126,7 +129,8 @@ typedef struct {
                                        src_rec; needs records).  Group g = (b*N + u)*T + st holds the records
                                        of source view u of asset b whose first kept tap lies in tile st:
                                        entries [g ? src_ptr[g-1] : 0, src_ptr[g]) of src_rec.  Sparse steps
-                                       with C >= 8 then apply the records per source tile (same results). */
+                                       with C >= 8 whose workspace has no room for the increment plane
+                                       then apply the records per source tile (same results). */
     int32_t* src_rec;               /* device [max_records][2] i32, 8-byte aligned, or NULL: entries
                                        (record index, target view v); their order within a group is not
                                        specified */
@@ -199,9 +203,15 @@ int geocache_build_corr(geocache_corr* corr, void* stream);
 int geocache_corr_record_count(geocache_corr* corr, int64_t* count, void* stream);
 
 /* --------------------------------------------------------------------------
- * geocache_transport_workspace -- number of floats of workspace that
- * geocache_transport_step needs for `corr` with C channels (0 unless
- * corr->mode is GEOCACHE_CORR_SPARSE, then max_records * C).  Host only.
+ * geocache_transport_workspace -- number of floats of workspace to give
+ * geocache_transport_step for `corr` with C channels: 0 unless corr->mode is
+ * GEOCACHE_CORR_SPARSE; then max_records * C (the minimum a step with a < N
+ * accepts), plus for C >= 8 room for the anchors' increment plane of any
+ * a < N, B * (N-1) * 4*ceil(C/4) * H * W floats.  A step with C >= 8 whose
+ * workspace holds max_records * C + B * a * 4*ceil(C/4) * H * W floats
+ * writes the plane and gathers the increments from it (faster); with less it
+ * applies the records into workspace rows.  Both give the same bits.  Host
+ * only.
  * ------------------------------------------------------------------------ */
 int64_t geocache_transport_workspace(const geocache_corr* corr, int C);
 
@@ -228,9 +238,12 @@ int64_t geocache_transport_workspace(const geocache_corr* corr, int C);
  *             view (bf16 stores round to nearest even); x_next may equal x_t.
  *             Ignored when recon is NULL.
  *   C         1 <= C <= GEOCACHE_MAX_CHANNELS.
- *   workspace device f32 scratch of at least geocache_transport_workspace(corr, C)
- *             floats (NULL when that is 0); its contents are not preserved
- *             between calls, and calls sharing a workspace must not overlap.
+ *   workspace device f32 scratch, 16-byte aligned, of workspace_floats floats:
+ *             in sparse mode with a < N at least max_records * C
+ *             (geocache_transport_workspace(corr, C) selects the fastest
+ *             path); NULL when no scratch is needed.  Its contents are not
+ *             preserved between calls, and calls sharing a workspace must not
+ *             overlap.
  * corr must have been filled by geocache_build_corr (tau; idx/w in
  * GEOCACHE_CORR_TABLE mode; keep in GEOCACHE_CORR_MASK mode; keep, tile_ptr
  * and records in GEOCACHE_CORR_SPARSE mode).
@@ -449,9 +462,10 @@ int geocache_debug_set_wait(uint64_t limit_ns, int drop_first_copy);
  * (16 MiB) in the library's device image, present on every device that loads
  * the library until the process exits.
  *  - A step that needs more scratch (a sparse-mode step with a < N whose
- *    geocache_transport_workspace(corr, C) exceeds the array) is rejected
- *    with GEOCACHE_ESHAPE; steps that need none (a == N, other modes) are
- *    always accepted.
+ *    max_records * C exceeds the array) is rejected with GEOCACHE_ESHAPE;
+ *    steps that need none (a == N, other modes) are always accepted.  The
+ *    whole array is passed as the workspace, so a step with C >= 8 takes
+ *    the increment-plane path when the array also holds the plane.
  *  - The first call on each device looks up the array's device address with
  *    that device current; make that first call before any stream capture.
  *    The address is kept for the life of the process, so the entry point

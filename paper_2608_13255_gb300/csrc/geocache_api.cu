@@ -231,7 +231,11 @@ int geocache_corr_record_count(geocache_corr* c, int64_t* count, void* stream) {
 
 int64_t geocache_transport_workspace(const geocache_corr* c, int C) {
     if (!c || C < 1 || c->mode != GEOCACHE_CORR_SPARSE || c->max_records < 0) return 0;
-    return c->max_records * (int64_t)C;
+    int64_t n = c->max_records * (int64_t)C;
+    // room for the anchors' increment plane of any step with a < N
+    if (C >= geocache::kPlaneMinChannels && c->N > 1)
+        n += geocache::plane_floats(c->B, c->N - 1, C, (long long)c->H * c->W);
+    return n;
 }
 
 int geocache_transport_step(const geocache_corr* c, const int32_t* anchors, int a, int C,
@@ -325,6 +329,7 @@ int geocache_transport_step_update(const geocache_corr* c, geocache_update updat
     t.src_ptr = c->mode == GEOCACHE_CORR_SPARSE ? c->src_ptr : nullptr;
     t.src_rec = c->mode == GEOCACHE_CORR_SPARSE ? c->src_rec : nullptr;
     t.workspace = workspace;
+    t.workspace_floats = workspace ? workspace_floats : 0;
     t.x0_new = x0_anchor_new; t.x0_prev = x0_prev; t.x0_out = x0_out;
     t.x_t = x_t; t.x_next = x_next; t.pred_out = recon ? recon->pred_out : nullptr;
     t.coef = coef;

@@ -51,7 +51,17 @@ struct TransportArgs {
     int32_t anchors[GEOCACHE_MAX_VIEWS];
     int32_t slot_of[GEOCACHE_MAX_VIEWS];   // slot in `anchors`, -1 for non-anchors
     int32_t others[GEOCACHE_MAX_VIEWS];    // the views outside the anchor set, ascending
+    long long workspace_floats;            // size of `workspace` (0 without one)
 };
+
+// The sparse step with wide latents (C >= kPlaneMinChannels) keeps the
+// anchors' increments as a plane [b][anchor slot][channel group][token] x 4
+// channels in the workspace, after room for max_records * C floats: it is
+// used when the workspace holds both (see geocache_transport_workspace).
+constexpr int kPlaneMinChannels = 8;
+inline long long plane_floats(long long B, long long a, int C, long long HW) {
+    return B * a * (long long)((C + 3) / 4) * 4 * HW;
+}
 
 struct RowAnchors {
     int32_t v[GEOCACHE_MAX_VIEWS];

@@ -1329,6 +1329,11 @@ template <typename T>
 constexpr int kPhaseABlocks = sizeof(T) == 2 ? 6 : 1;
 template <typename T>
 constexpr int kPhaseBBlocks = sizeof(T) == 2 ? 5 : 1;
+// The increment-plane kernels (wide latents) at 4 resident CTAs per SM: no
+// spills (62 / 64 registers); at 5 or 6 the spills cost more than the
+// residency gains.
+constexpr int kPlaneABlocks = 4;
+constexpr int kPlaneBBlocks = 4;
 
 template <typename T, int K, bool VEC, bool COPY>
 __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_kernel(const TransportArgs args, int n_apply,
@@ -1364,9 +1369,12 @@ __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_ker
 // Phase B: one CTA per (tile, group of 4 channels) of a view; blockIdx.y <
 // N - a: views outside the anchor set (fold the tile's increments);
 // blockIdx.y >= N - a: anchor views (only for an in-place cache update, see
-// phase A).
-template <typename T, bool VEC, bool COPY>
-__global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_kernel(const TransportArgs args, int n_cg) {
+// phase A).  PK = 0: each record's increment is its workspace row, written
+// by phase A's apply; PK = K: it is formed here from the anchors' increment
+// plane, sum_k w_k increment[q_k] in tap order (the same terms in the same
+// order as the applies, so the same bits).
+template <typename T, bool VEC, bool COPY, int PK>
+__global__ void __launch_bounds__(kThreads, PK ? kPlaneBBlocks : kPhaseBBlocks<T>) sparse_phase_b_kernel(const TransportArgs args, int n_cg) {
     __shared__ float s_acc[kTileTokens][4];
     __shared__ __align__(4) uint8_t s_n[kTileTokens];
     __shared__ int s_r0[GEOCACHE_MAX_VIEWS], s_cnt[GEOCACHE_MAX_VIEWS];
@@ -1429,15 +1437,37 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
             int s2 = 0, jj = j;
             while (jj >= s_cnt[s2]) jj -= s_cnt[s2++];
             const int r = s_r0[s2] + jj;
-            lp = (__ldg(&args.records[r].token_mask) & 0x0fffffff) - tile0;
-            const float* w = args.workspace + (size_t)r * C + cg;
-            if (cn == 4 && C % 4 == 0) {
-                const float4 wq = *reinterpret_cast<const float4*>(w);
-                g[0] = wq.x; g[1] = wq.y; g[2] = wq.z; g[3] = wq.w;
-            } else {
+            if (PK) {  // sum_k w_k increment[q_k] in tap order, from the anchor's increment plane
+                const int4 rec = __ldg(reinterpret_cast<const int4*>(args.records) + r);
+                lp = (rec.x & 0x0fffffff) - tile0;
+                Taps tp;
+                taps_from_record<PK ? PK : 1>((int)((uint32_t)rec.x >> 28), rec.y, __int_as_float(rec.z),
+                                              __int_as_float(rec.w), args.W, tp);
+                const float4* d = reinterpret_cast<const float4*>(args.workspace) +
+                                  (((size_t)b * a + s2) * n_cg + cg / 4) * (size_t)HW;
+                float4 dq[PK ? PK : 1];
 #pragma unroll
-                for (int c = 0; c < 4; ++c)
-                    if (c < cn) g[c] = w[c];
+                for (int kk = 0; kk < (PK ? PK : 1); ++kk)
+                    dq[kk] = tp.q[kk] >= 0 ? __ldg(d + tp.q[kk]) : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int kk = 0; kk < (PK ? PK : 1); ++kk) {
+                    if (tp.q[kk] < 0) continue;
+                    g[0] = __fmaf_rn(tp.w[kk], dq[kk].x, g[0]);
+                    g[1] = __fmaf_rn(tp.w[kk], dq[kk].y, g[1]);
+                    g[2] = __fmaf_rn(tp.w[kk], dq[kk].z, g[2]);
+                    g[3] = __fmaf_rn(tp.w[kk], dq[kk].w, g[3]);
+                }
+            } else {
+                lp = (__ldg(&args.records[r].token_mask) & 0x0fffffff) - tile0;
+                const float* w = args.workspace + (size_t)r * C + cg;
+                if (cn == 4 && C % 4 == 0) {
+                    const float4 wq = *reinterpret_cast<const float4*>(w);
+                    g[0] = wq.x; g[1] = wq.y; g[2] = wq.z; g[3] = wq.w;
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 4; ++c)
+                        if (c < cn) g[c] = w[c];
+                }
             }
             s_mine = s2;
         }
@@ -1466,6 +1496,73 @@ __global__ void __launch_bounds__(kThreads, kPhaseBBlocks<T>) sparse_phase_b_ker
         const uint32_t n4 = *reinterpret_cast<const uint32_t*>(s_n + 4 * t);
         if (n4) q.template fold4<COPY>(s_acc, n4, 4 * t);
         q.store(args, b, v, p0, cnt, cg, cn);
+    }
+}
+
+// Phase A with the anchors' increment plane (wide latents): one CTA per
+// (asset, anchor slot, tile, group of 4 channels) streams the anchor tile
+// (x0(t) = x0_new and the reconstruction) and writes the tile's increment
+// x0_new - x0(t-1) (x0_new itself under the value copy) to the plane
+// [b][slot][channel group][token] x 4 channels in the workspace, where phase
+// B gathers it at the records' taps.  Each element is read before the same
+// thread writes it, so the stream is also correct for an in-place update.
+template <typename T, bool VEC, bool COPY>
+__global__ void __launch_bounds__(kThreads, kPlaneABlocks) sparse_phase_a_plane_kernel(const TransportArgs args,
+                                                                                         int n_cg) {
+    pdl_launch_dependents();
+    const int HW = args.H * args.W;
+    const int n_tiles = tiles_per_view_dev(args.H, args.W);
+    long long k = blockIdx.x;
+    const int cgi = (int)(k % n_cg);
+    k /= n_cg;
+    const int tile = (int)(k % n_tiles);
+    k /= n_tiles;
+    const int slot = (int)(k % args.a);
+    const int b = (int)(k / args.a);
+    const int p0 = tile * kTileTokens + 4 * threadIdx.x;
+    if (p0 >= HW) return;
+    const int cnt = HW - p0 < 4 ? HW - p0 : 4;
+    const int cg = cgi * 4;
+    const int cn = args.C - cg < 4 ? args.C - cg : 4;
+    const size_t plane = (size_t)HW;
+    const int u = args.anchors[slot];
+    const float* xn = args.x0_new + ((size_t)b * args.a + slot) * args.C * plane;
+    const float* xp = args.x0_prev + ((size_t)b * args.N + u) * args.C * plane;
+    const size_t view_base = ((size_t)b * args.N + u) * args.C * plane;
+    const T* xt_p = static_cast<const T*>(args.x_t);
+    T* xn_p = static_cast<T*>(args.x_next);
+    float dn[4][4], pv[4][4];
+    typename Lat4<T>::Raw xr[4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        if (c >= cn) break;
+        const size_t e = (size_t)(cg + c) * plane + p0;
+        Lat4<float>::load(xn, e, cnt, VEC, dn[c]);
+        if (!COPY) Lat4<float>::load(xp, e, cnt, VEC, pv[c]);
+        if (args.coef.enabled) xr[c] = Lat4<T>::load_raw(xt_p, view_base + e, cnt, VEC);
+    }
+    float dd[4][4];
+#pragma unroll
+    for (int c = 0; c < 4; ++c)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) dd[c][i] = c < cn ? (COPY ? dn[c][i] : __fsub_rn(dn[c][i], pv[c][i])) : 0.0f;
+    float4* d = reinterpret_cast<float4*>(args.workspace) + (((size_t)b * args.a + slot) * n_cg + cgi) * plane + p0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        if (i < cnt) d[i] = make_float4(dd[0][i], dd[1][i], dd[2][i], dd[3][i]);
+#pragma unroll
+    for (int c = 0; c < 4; ++c) {
+        if (c >= cn) break;
+        const size_t e = view_base + (size_t)(cg + c) * plane + p0;
+        Lat4<float>::store(args.x0_out, e, cnt, VEC, dn[c]);
+        if (args.coef.enabled) {
+            float x[4], yv[4], pr[4];
+            Lat4<T>::unpack(xr[c], x);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) yv[i] = recon_one(args.coef, x[i], dn[c][i], pr[i]);
+            Lat4<T>::store(xn_p, e, cnt, VEC, yv);
+            if (args.pred_out) Lat4<float>::store(args.pred_out, e, cnt, VEC, pr);
+        }
     }
 }
 
@@ -1607,11 +1704,27 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
     const bool vec = (HW % 4 == 0) && (al % 16 == 0);
     const bool in_place = t.x0_out == t.x0_prev;
     const bool copy = t.update == GEOCACHE_UPDATE_COPY;
-    // phase A by source tile when the corr has a source index, the latents are
-    // wide and the staged span (tile + W + 1 tokens) fits
-    const bool by_source = t.a < t.N && t.src_ptr && t.src_rec && t.C >= kSrcMinChannels && t.W + 1 <= kTileTokens;
+    // wide latents: the anchors' increment plane when the workspace holds it
+    // beside max_records * C floats, else phase A by source tile when the
+    // corr has a source index and the staged span (tile + W + 1 tokens)
+    // fits, else the record-parallel apply
+    const long long n_plane = plane_floats(t.B, t.a, t.C, HW);
+    const bool by_plane = t.a < t.N && t.C >= kPlaneMinChannels && t.workspace &&
+                          t.workspace_floats >= t.max_records * (long long)t.C + n_plane;
+    const bool by_source = !by_plane && t.a < t.N && t.src_ptr && t.src_rec && t.C >= kSrcMinChannels &&
+                           t.W + 1 <= kTileTokens;
     bool phase_a = false;
-    if (by_source) {
+    if (by_plane) {
+        const long long g = (long long)t.B * t.a * n_tiles * n_cg;
+        if (g > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+        if (vec && !copy) sparse_phase_a_plane_kernel<T, true, false><<<(unsigned)g, kThreads, 0, s>>>(t, n_cg);
+        else if (vec) sparse_phase_a_plane_kernel<T, true, true><<<(unsigned)g, kThreads, 0, s>>>(t, n_cg);
+        else if (!copy) sparse_phase_a_plane_kernel<T, false, false><<<(unsigned)g, kThreads, 0, s>>>(t, n_cg);
+        else sparse_phase_a_plane_kernel<T, false, true><<<(unsigned)g, kThreads, 0, s>>>(t, n_cg);
+        cudaError_t e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+        phase_a = true;
+    } else if (by_source) {
         const long long g = (long long)t.B * t.a * n_tiles * n_cg;
         if (g > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
         const size_t dyn = (size_t)(kTileTokens + t.W + 1) * sizeof(float4);
@@ -1647,7 +1760,9 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
             phase_a = true;
         }
     }
-    const int gy = (t.N - t.a) + (in_place ? t.a : 0);
+    // an in-place update streams the anchor views after the wait, except with
+    // the plane (its phase A reads each anchor element before writing it)
+    const int gy = (t.N - t.a) + (in_place && !by_plane ? t.a : 0);
     if (gy > 0) {
         if ((long long)n_tiles * n_cg > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
         cudaLaunchConfig_t cfg = {};
@@ -1661,10 +1776,17 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
         cfg.attrs = attr;
         cfg.numAttrs = 1;
         cudaError_t e;
-        if (vec && !copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, false>, t, n_cg);
-        else if (vec) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, true>, t, n_cg);
-        else if (!copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, false>, t, n_cg);
-        else e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, true>, t, n_cg);
+        if (by_plane) {
+            if (vec && !copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, false, K>, t, n_cg);
+            else if (vec) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, true, K>, t, n_cg);
+            else if (!copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, false, K>, t, n_cg);
+            else e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, true, K>, t, n_cg);
+        } else {
+            if (vec && !copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, false, 0>, t, n_cg);
+            else if (vec) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, true, 0>, t, n_cg);
+            else if (!copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, false, 0>, t, n_cg);
+            else e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, true, 0>, t, n_cg);
+        }
         if (e != cudaSuccess) return e;
     }
     return cudaGetLastError();

@@ -51,8 +51,12 @@ extern "C" int geocache_transport_step_noalloc(const geocache_corr* corr, const 
                                                const float* x0_anchor_new, const float* x0_prev, float* x0_out,
                                                const void* x_t, void* x_next, geocache_dtype lat_dtype,
                                                const geocache_recon* recon, void* stream) {
-    // only a sparse-mode step with a view outside the anchor set uses scratch
-    const int64_t need = (corr && a < corr->N) ? geocache_transport_workspace(corr, C) : 0;
+    // only a sparse-mode step with a view outside the anchor set uses scratch,
+    // at least max_records * C floats (the whole array is passed, so the
+    // increment-plane path runs whenever the array also holds the plane)
+    const int64_t need = (corr && a < corr->N && corr->mode == GEOCACHE_CORR_SPARSE && corr->max_records > 0 && C > 0)
+                             ? corr->max_records * (int64_t)C
+                             : 0;
     if (need > kNoallocFloats)
         return geocache::set_error(GEOCACHE_ESHAPE,
                                    "geocache_transport_step_noalloc: this step needs %lld floats of scratch but the "

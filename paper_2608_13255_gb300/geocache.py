@@ -197,7 +197,12 @@ class CorrHandle:
         return self._keep.get("keep")
 
     def workspace_floats(self, C: int) -> int:
+        """Workspace floats that select the fastest sparse path for C channels."""
         return load().geocache_transport_workspace(ctypes.byref(self.c), int(C))
+
+    def min_workspace_floats(self, C: int) -> int:
+        """The smallest workspace a sparse step with a < N accepts (max_records * C)."""
+        return self.c.max_records * int(C) if self.c.mode == CORR_SPARSE else 0
 
 
 def tiles_per_view(H: int, W: int) -> int:
@@ -243,9 +248,10 @@ def build_sparse_corr(pos, valid, cams, K=4, tol_frac=0.01, tables=False, stream
                       source_index=False) -> CorrHandle:
     """Allocate and build the full correspondence state of a batch: tau, keep
     masks, the sparse form (count, then records), optionally the tables and
-    the source index (worth building for latents of 8 or more channels, whose
-    steps then apply the records per source tile).  Allocation happens here,
-    once per batch of assets, never per step."""
+    the source index (used by steps with 8 or more channels whose workspace
+    has no room for the anchors' increment plane: they then apply the records
+    per source tile).  Allocation happens here, once per batch of assets,
+    never per step."""
     B, N, H, W = valid.shape
     dev = pos.device
     tau = torch.zeros(B, dtype=torch.float32, device=dev)

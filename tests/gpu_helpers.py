@@ -170,5 +170,9 @@ class DeviceGeometry:
                             tol_frac=self.w.tol_frac, keep=self.keep, tile_ptr=self.tile_ptr, records=self.records,
                             mode=m, src_ptr=self.src_ptr if src else None, src_rec=self.src_rec if src else None)
 
-    def workspace(self, C):
-        return torch.empty(max(self.corr.workspace_floats(C), 4), dtype=torch.float32, device=self.pos.device)
+    def workspace(self, C, minimal=False):
+        """Scratch for a sparse step: the fastest path's size, or (minimal)
+        the smallest one a step accepts, max_records * C floats, which leaves
+        no room for the increment plane of wide latents."""
+        n = self.corr.min_workspace_floats(C) if minimal else self.corr.workspace_floats(C)
+        return torch.empty(max(n, 4), dtype=torch.float32, device=self.pos.device)

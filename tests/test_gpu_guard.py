@@ -83,12 +83,16 @@ def _geometry(gc, w, K=4, skew=0, records_frac=1.0):
     return corr, g, R, cap, (pos, valid, cams)
 
 
-@pytest.mark.parametrize("case", ["ragged_c5", "ragged_c18", "misaligned", "c3_k1"])
+@pytest.mark.parametrize("case", ["ragged_c5", "ragged_c18", "ragged_c18_src", "misaligned", "c3_k1"])
 def test_transport_writes_only_its_outputs(gc, case):
+    minimal_ws = False
     if case == "ragged_c5":  # 37 x 53 tokens: H*W = 1961, two tiles, a ragged quad; C = 5
         w, C, skew, K = synth.make_workload("batch128", B=2, H=37, W=53), 5, 0, 4
-    elif case == "ragged_c18":  # the same with C = 18: the source-tile apply, a partial last channel group
+    elif case == "ragged_c18":  # the same with C = 18: the increment plane, a partial last channel group
         w, C, skew, K = synth.make_workload("batch128", B=2, H=37, W=53), 18, 0, 4
+    elif case == "ragged_c18_src":  # C = 18 with the minimal workspace: the source-tile apply
+        w, C, skew, K = synth.make_workload("batch128", B=2, H=37, W=53), 18, 0, 4
+        minimal_ws = True
     elif case == "misaligned":  # 64 x 64 tokens, every buffer 4 bytes off a 16-byte boundary
         w, C, skew, K = synth.make_workload("hunyuan64"), 4, 4, 4
     else:
@@ -113,7 +117,8 @@ def test_transport_writes_only_its_outputs(gc, case):
         out = Guarded(shp, torch.float32, skew)
         xn = Guarded(shp, lat, skew)
         pred = Guarded(shp, torch.float32, skew)
-        ws = Guarded((max(c2.workspace_floats(C), 4),), torch.float32, 0)
+        nws = c2.min_workspace_floats(C) if minimal_ws else c2.workspace_floats(C)
+        ws = Guarded((max(nws, 4),), torch.float32, 0)
         r = gc.make_recon(p["sampler"], a_t=p.get("a_t", 0), a_prev=p.get("a_prev", 0), sigma=p.get("sigma", 0),
                           sigma_next=p.get("sigma_next", 0), pred_kind=pred_kind, pred_out=pred.t)
         d_prev = Guarded(shp, torch.float32, skew, torch.from_numpy(x0_prev))

@@ -88,7 +88,7 @@ def test_tables_bit_exact_k1(gc, workloads, name):
 
 
 def _run_step(gc, w, g, anchors, params, pred=None, mode="sparse", inplace=False, xinplace=False,
-              seed_extra=0, C=None):
+              seed_extra=0, C=None, minimal_ws=False):
     """One cached step on the GPU and in the oracle from the same inputs."""
     if C is not None and C != w.C:
         w = synth.Workload(**{**w.__dict__, "C": C})
@@ -105,7 +105,8 @@ def _run_step(gc, w, g, anchors, params, pred=None, mode="sparse", inplace=False
     r = gc.make_recon(params["sampler"], a_t=params.get("a_t", 0), a_prev=params.get("a_prev", 0),
                       sigma=params.get("sigma", 0), sigma_next=params.get("sigma_next", 0),
                       pred_kind=pred, pred_out=d_pred)
-    gc.transport_step(corr, anchors, w.C, d_new, d_prev, d_out, d_xt, d_xn, r, workspace=g.workspace(w.C))
+    gc.transport_step(corr, anchors, w.C, d_new, d_prev, d_out, d_xt, d_xn, r,
+                      workspace=g.workspace(w.C, minimal=minimal_ws))
     torch.cuda.synchronize()
     gc.device_status()
     tau_ref = oracle.tau(w.pos, w.valid, w.tol_frac)
@@ -491,17 +492,23 @@ def test_source_index_groups_every_record_once(gc, workloads, name):
 
 @pytest.mark.parametrize("C,update,inplace", [(16, "delta", False), (16, "delta", True), (20, "copy", False),
                                               (33, "delta", False), (8, "copy", True)])
-def test_source_tile_apply_equals_record_parallel_apply(gc, workloads, C, update, inplace):
-    # wide latents (C >= 8) apply the records per source tile when the corr
-    # has a source index: bitwise the results of the record-parallel apply, and
-    # the oracle's
+def test_wide_latent_paths_agree_bitwise(gc, workloads, C, update, inplace):
+    # wide latents (C >= 8) have three ways to form the records' increments:
+    # the anchors' increment plane (workspace with room for it), the
+    # source-tile apply (minimal workspace, corr with a source index) and the
+    # record-parallel apply (minimal workspace, no index).  All three give the
+    # same bits, and the oracle's results.
     w = workloads("ring12_128") if C == 16 else workloads("solids96")
     w = synth.Workload(**{**w.__dict__, "C": C})
     g = DeviceGeometry(w, K=w.K, tables=False)
     anchors = oracle.rotate_anchors(w.N, w.a, 1)
     params = synth.recon_params(w, 8)
     outs = {}
-    for mode in ("sparse", "sparse_plain"):
+    for path, mode, minimal in (("plane", "sparse_plain", False), ("source_tile", "sparse", True),
+                                ("record", "sparse_plain", True)):
+        ws = g.workspace(C, minimal=minimal)
+        if not minimal:  # room for max_records * C floats and the plane
+            assert ws.numel() >= g.corr.min_workspace_floats(C) + len(anchors) * w.B * -(-C // 4) * 4 * w.H * w.W
         x0_prev, x0_new, xt32 = step_inputs(w, 3, anchors)
         xt64, xt = latent_values(xt32, w)
         d_prev, d_new, d_xt = torch.from_numpy(x0_prev).cuda(), torch.from_numpy(x0_new).cuda(), xt.cuda()
@@ -509,24 +516,26 @@ def test_source_tile_apply_equals_record_parallel_apply(gc, workloads, C, update
         d_xn = d_xt if inplace else torch.empty_like(d_xt)
         r = gc.make_recon(params["sampler"], a_t=params.get("a_t", 0), a_prev=params.get("a_prev", 0),
                           sigma=params.get("sigma", 0), sigma_next=params.get("sigma_next", 0))
-        gc.transport_step(g.corr_for(mode), anchors, C, d_new, d_prev, d_out, d_xt, d_xn, r,
-                          workspace=g.workspace(C), update=update)
+        gc.transport_step(g.corr_for(mode), anchors, C, d_new, d_prev, d_out, d_xt, d_xn, r, workspace=ws,
+                          update=update)
         torch.cuda.synchronize()
         gc.device_status()
-        outs[mode] = (d_out.cpu().numpy(), d_xn.cpu().view(torch.int16).numpy())
-    np.testing.assert_array_equal(outs["sparse"][0], outs["sparse_plain"][0])
-    np.testing.assert_array_equal(outs["sparse"][1], outs["sparse_plain"][1])
+        outs[path] = (d_out.cpu().numpy(), d_xn.cpu().view(torch.int16).numpy())
+    for path in ("source_tile", "record"):
+        np.testing.assert_array_equal(outs[path][0], outs["plane"][0])
+        np.testing.assert_array_equal(outs[path][1], outs["plane"][1])
     tau = oracle.tau(w.pos, w.valid, w.tol_frac)
     ref_x0, ref_xn, _ = oracle.transport_step(anchors, x0_new, x0_prev, K=w.K, geom=(w.pos, w.valid, w.cams, tau),
                                               x_t=xt64, recon=recon_kw(params), update=update)
-    assert_f32_close(outs["sparse"][0], ref_x0, what="x0")
-    assert_bf16_close(outs["sparse"][1].view(np.uint16), ref_xn, what="x_next")
+    assert_f32_close(outs["plane"][0], ref_x0, what="x0")
+    assert_bf16_close(outs["plane"][1].view(np.uint16), ref_xn, what="x_next")
 
 
 def test_wide_views_fall_back_to_the_record_parallel_apply(gc):
     # W + 1 > 1024 tokens: the staged span of a source tile would not fit, so a
-    # step with a source index applies the records record-parallel; results
-    # equal the oracle's
+    # step with a source index and a minimal workspace applies the records
+    # record-parallel; with room for the increment plane (no span limit) it
+    # takes the plane.  Both equal the oracle's results.
     H, W = 16, 1040
     w = synth.make_workload("solids96", H=H, W=W)
     cams = np.stack([synth.look_at_camera(az, el, W, W) for az, el in synth.hunyuan_layout()])
@@ -536,4 +545,6 @@ def test_wide_views_fall_back_to_the_record_parallel_apply(gc):
                           "valid": valid[None]})
     g = DeviceGeometry(w, K=4, tables=False)
     assert g.n_records > 100
-    _run_step(gc, w, g, [0, 2, 4], synth.recon_params(w, 5))
+    _, _, x0_min, _ = _run_step(gc, w, g, [0, 2, 4], synth.recon_params(w, 5), minimal_ws=True)
+    _, _, x0_plane, _ = _run_step(gc, w, g, [0, 2, 4], synth.recon_params(w, 5))
+    np.testing.assert_array_equal(x0_min, x0_plane)
