@@ -1247,6 +1247,30 @@ __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepc
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 
+// Quotient by a divisor fixed for a launch, as a multiply-high and a shift
+// (Granlund and Montgomery, division by invariant integers using
+// multiplication): with l = ceil(log2 d) and m = floor(2^32 (2^l - d) / d) + 1,
+// n / d = (umulhi(m, n) + n) >> l for 0 <= n < 2^31.  The CTAs of a launch
+// split their block index into (asset, view, tile, channel group, ...) with
+// these instead of integer divisions.
+struct FastDiv {
+    uint32_t d, m, l;
+    __device__ __forceinline__ uint32_t quo(uint32_t n) const { return (__umulhi(m, n) + n) >> l; }
+};
+static FastDiv make_fastdiv(uint32_t d) {
+    FastDiv f{d, 0u, 0u};
+    while ((1ull << f.l) < d) ++f.l;
+    f.m = (uint32_t)(((1ull << 32) * ((1ull << f.l) - d)) / d + 1);
+    return f;
+}
+
+// Grid shape of a sparse step's launches and the divisors that split it.
+struct SparseGrid {
+    int n_cg, n_tiles, n_slices, n_stream, n_total;
+    int small;  // n_total * n_stream < 2^31: the interleave's quotients in 32 bits
+    FastDiv cg, tiles, a, na, slices, total;
+};
+
 // Tile offset i of the sparse form clamped to the records that exist, [0,
 // cap]: a build whose records overflowed the capacity or the int32 offsets
 // is flagged in the status word, and the transport then reads only records
@@ -1260,13 +1284,16 @@ __device__ __forceinline__ int record_offset(const int32_t* __restrict__ tile_pt
 // records), channels [cg, cg + 4).  COPY: the value-copy ablation (no x0(t-1)
 // gathers).
 template <int K, bool COPY>
-__device__ __forceinline__ void apply_records(const TransportArgs& args, int pair_id, int slice, int n_slices, int cg) {
+__device__ __forceinline__ void apply_records(const TransportArgs& args, const SparseGrid& g, int pair_id, int slice,
+                                              int cg) {
     const int N = args.N, C = args.C, a = args.a;
     const int HW = args.H * args.W;
-    const int T = tiles_per_view_dev(args.H, args.W);
-    const int s2 = pair_id % a;
-    const int vi = (pair_id / a) % (N - a);
-    const int b = pair_id / (a * (N - a));
+    const int T = g.n_tiles;
+    const int n_slices = g.n_slices;
+    const int pa = (int)g.a.quo((uint32_t)pair_id);
+    const int s2 = pair_id - pa * a;
+    const int b = (int)g.na.quo((uint32_t)pa);
+    const int vi = pa - b * (N - a);
     const int v = args.others[vi];
     const int u = args.anchors[s2];
     const size_t pair = ((size_t)b * N + v) * N + u;
@@ -1336,24 +1363,31 @@ constexpr int kPlaneABlocks = 4;
 constexpr int kPlaneBBlocks = 4;
 
 template <typename T, int K, bool VEC, bool COPY>
-__global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_kernel(const TransportArgs args, int n_apply,
-                                                                  int n_stream, int n_slices, int n_cg) {
+__global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_kernel(const TransportArgs args,
+                                                                                    const SparseGrid g) {
     pdl_launch_dependents();
-    const long long total = (long long)n_apply + n_stream;
-    const long long k = blockIdx.x;
-    const int s_before = (int)(k * n_stream / total);
-    const bool is_stream = (int)((k + 1) * n_stream / total) > s_before;
-    if (!is_stream) {
+    const uint32_t k = blockIdx.x;
+    int s_before, s_next;
+    if (g.small) {
+        s_before = (int)g.total.quo(k * (uint32_t)g.n_stream);
+        s_next = (int)g.total.quo((k + 1) * (uint32_t)g.n_stream);
+    } else {
+        s_before = (int)((long long)k * g.n_stream / g.n_total);
+        s_next = (int)(((long long)k + 1) * g.n_stream / g.n_total);
+    }
+    if (s_next == s_before) {  // a record-apply CTA
         const int ai = (int)k - s_before;
-        const int aj = ai / n_cg;
-        apply_records<K, COPY>(args, aj / n_slices, aj % n_slices, n_slices, (ai % n_cg) * 4);
+        const int aj = (int)g.cg.quo((uint32_t)ai);
+        const int pair = (int)g.slices.quo((uint32_t)aj);
+        apply_records<K, COPY>(args, g, pair, aj - pair * g.n_slices, (ai - aj * g.n_cg) * 4);
         return;
     }
-    const int n_tiles = tiles_per_view_dev(args.H, args.W);
-    const int cg = (s_before % n_cg) * 4;
-    const int tile = (s_before / n_cg) % n_tiles;
-    const int slot = (s_before / (n_cg * n_tiles)) % args.a;
-    const int b = s_before / (n_cg * n_tiles * args.a);
+    const int q1 = (int)g.cg.quo((uint32_t)s_before);
+    const int cg = (s_before - q1 * g.n_cg) * 4;
+    const int q2 = (int)g.tiles.quo((uint32_t)q1);
+    const int tile = q1 - q2 * g.n_tiles;
+    const int b = (int)g.a.quo((uint32_t)q2);
+    const int slot = q2 - b * args.a;
     const int v = args.anchors[slot];
     const int HW = args.H * args.W;
     const int tile0 = tile * kTileTokens;
@@ -1374,13 +1408,14 @@ __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_ker
 // plane, sum_k w_k increment[q_k] in tap order (the same terms in the same
 // order as the applies, so the same bits).
 template <typename T, bool VEC, bool COPY, int PK>
-__global__ void __launch_bounds__(kThreads, PK ? kPlaneBBlocks : kPhaseBBlocks<T>) sparse_phase_b_kernel(const TransportArgs args, int n_cg) {
+__global__ void __launch_bounds__(kThreads, PK ? kPlaneBBlocks : kPhaseBBlocks<T>) sparse_phase_b_kernel(const TransportArgs args, const SparseGrid g) {
     __shared__ float s_acc[kTileTokens][4];
     __shared__ __align__(4) uint8_t s_n[kTileTokens];
     __shared__ int s_r0[GEOCACHE_MAX_VIEWS], s_cnt[GEOCACHE_MAX_VIEWS];
     const int HW = args.H * args.W;
     const int T_tiles = tiles_per_view_dev(args.H, args.W);
-    const int tile = blockIdx.x / n_cg, cg = (blockIdx.x % n_cg) * 4, b = blockIdx.z;
+    const int n_cg = g.n_cg;
+    const int tile = (int)g.cg.quo(blockIdx.x), cg = ((int)blockIdx.x - tile * n_cg) * 4, b = blockIdx.z;
     const int N = args.N, C = args.C, a = args.a;
     const int cn = C - cg < 4 ? C - cg : 4;
     const int tile0 = tile * kTileTokens;
@@ -1508,17 +1543,16 @@ __global__ void __launch_bounds__(kThreads, PK ? kPlaneBBlocks : kPhaseBBlocks<T
 // thread writes it, so the stream is also correct for an in-place update.
 template <typename T, bool VEC, bool COPY>
 __global__ void __launch_bounds__(kThreads, kPlaneABlocks) sparse_phase_a_plane_kernel(const TransportArgs args,
-                                                                                         int n_cg) {
+                                                                                         const SparseGrid g) {
     pdl_launch_dependents();
     const int HW = args.H * args.W;
-    const int n_tiles = tiles_per_view_dev(args.H, args.W);
-    long long k = blockIdx.x;
-    const int cgi = (int)(k % n_cg);
-    k /= n_cg;
-    const int tile = (int)(k % n_tiles);
-    k /= n_tiles;
-    const int slot = (int)(k % args.a);
-    const int b = (int)(k / args.a);
+    const int n_cg = g.n_cg;
+    const int q1 = (int)g.cg.quo(blockIdx.x);
+    const int cgi = (int)blockIdx.x - q1 * n_cg;
+    const int q2 = (int)g.tiles.quo((uint32_t)q1);
+    const int tile = q1 - q2 * g.n_tiles;
+    const int b = (int)g.a.quo((uint32_t)q2);
+    const int slot = q2 - b * args.a;
     const int p0 = tile * kTileTokens + 4 * threadIdx.x;
     if (p0 >= HW) return;
     const int cnt = HW - p0 < 4 ? HW - p0 : 4;
@@ -1579,19 +1613,18 @@ __global__ void __launch_bounds__(kThreads, kPlaneABlocks) sparse_phase_a_plane_
 // of the anchor tile.
 template <typename T, int K, bool COPY>
 __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_src_kernel(const TransportArgs args,
-                                                                                       int n_cg, int stream) {
+                                                                                       const SparseGrid g, int stream) {
     pdl_launch_dependents();
     extern __shared__ __align__(16) float4 s_d[];  // [kTileTokens + W + 1] tokens x 4 channels
     const int HW = args.H * args.W, W = args.W;
     const int N = args.N, C = args.C, a = args.a;
-    const int n_tiles = tiles_per_view_dev(args.H, args.W);
-    long long k = blockIdx.x;
-    const int cg = (int)(k % n_cg) * 4;
-    k /= n_cg;
-    const int st = (int)(k % n_tiles);
-    k /= n_tiles;
-    const int slot = (int)(k % a);
-    const int b = (int)(k / a);
+    const int n_tiles = g.n_tiles;
+    const int q1 = (int)g.cg.quo(blockIdx.x);
+    const int cg = ((int)blockIdx.x - q1 * g.n_cg) * 4;
+    const int q2 = (int)g.tiles.quo((uint32_t)q1);
+    const int st = q1 - q2 * n_tiles;
+    const int b = (int)g.a.quo((uint32_t)q2);
+    const int slot = q2 - b * a;
     const int u = args.anchors[slot];
     const int cn = C - cg < 4 ? C - cg : 4;
     const size_t plane = (size_t)HW;
@@ -1708,6 +1741,13 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
     // beside max_records * C floats, else phase A by source tile when the
     // corr has a source index and the staged span (tile + W + 1 tokens)
     // fits, else the record-parallel apply
+    SparseGrid sg{};
+    sg.n_cg = n_cg;
+    sg.n_tiles = n_tiles;
+    sg.cg = make_fastdiv((uint32_t)n_cg);
+    sg.tiles = make_fastdiv((uint32_t)n_tiles);
+    sg.a = make_fastdiv((uint32_t)t.a);
+    sg.na = make_fastdiv((uint32_t)(t.N > t.a ? t.N - t.a : 1));
     const long long n_plane = plane_floats(t.B, t.a, t.C, HW);
     const bool by_plane = t.a < t.N && t.C >= kPlaneMinChannels && t.workspace &&
                           t.workspace_floats >= t.max_records * (long long)t.C + n_plane;
@@ -1717,10 +1757,10 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
     if (by_plane) {
         const long long g = (long long)t.B * t.a * n_tiles * n_cg;
         if (g > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-        if (vec && !copy) sparse_phase_a_plane_kernel<T, true, false><<<(unsigned)g, kThreads, 0, s>>>(t, n_cg);
-        else if (vec) sparse_phase_a_plane_kernel<T, true, true><<<(unsigned)g, kThreads, 0, s>>>(t, n_cg);
-        else if (!copy) sparse_phase_a_plane_kernel<T, false, false><<<(unsigned)g, kThreads, 0, s>>>(t, n_cg);
-        else sparse_phase_a_plane_kernel<T, false, true><<<(unsigned)g, kThreads, 0, s>>>(t, n_cg);
+        if (vec && !copy) sparse_phase_a_plane_kernel<T, true, false><<<(unsigned)g, kThreads, 0, s>>>(t, sg);
+        else if (vec) sparse_phase_a_plane_kernel<T, true, true><<<(unsigned)g, kThreads, 0, s>>>(t, sg);
+        else if (!copy) sparse_phase_a_plane_kernel<T, false, false><<<(unsigned)g, kThreads, 0, s>>>(t, sg);
+        else sparse_phase_a_plane_kernel<T, false, true><<<(unsigned)g, kThreads, 0, s>>>(t, sg);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         phase_a = true;
@@ -1729,9 +1769,9 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
         if (g > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
         const size_t dyn = (size_t)(kTileTokens + t.W + 1) * sizeof(float4);
         if (!copy)
-            sparse_phase_a_src_kernel<T, K, false><<<(unsigned)g, kThreads, dyn, s>>>(t, n_cg, in_place ? 0 : 1);
+            sparse_phase_a_src_kernel<T, K, false><<<(unsigned)g, kThreads, dyn, s>>>(t, sg, in_place ? 0 : 1);
         else
-            sparse_phase_a_src_kernel<T, K, true><<<(unsigned)g, kThreads, dyn, s>>>(t, n_cg, in_place ? 0 : 1);
+            sparse_phase_a_src_kernel<T, K, true><<<(unsigned)g, kThreads, dyn, s>>>(t, sg, in_place ? 0 : 1);
         cudaError_t e = cudaGetLastError();
         if (e != cudaSuccess) return e;
         phase_a = true;
@@ -1746,15 +1786,20 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
         if (n_apply + n_stream > 0) {
             if (n_apply + n_stream > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
             const unsigned g = (unsigned)(n_apply + n_stream);
-            const int ns = (int)n_slices;
+            sg.n_slices = (int)n_slices;
+            sg.slices = make_fastdiv((uint32_t)n_slices);
+            sg.n_stream = (int)n_stream;
+            sg.n_total = (int)g;
+            sg.total = make_fastdiv(g);
+            sg.small = (long long)g * n_stream < 0x80000000LL;
             if (vec && !copy)
-                sparse_phase_a_kernel<T, K, true, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, ns, n_cg);
+                sparse_phase_a_kernel<T, K, true, false><<<g, kThreads, 0, s>>>(t, sg);
             else if (vec)
-                sparse_phase_a_kernel<T, K, true, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, ns, n_cg);
+                sparse_phase_a_kernel<T, K, true, true><<<g, kThreads, 0, s>>>(t, sg);
             else if (!copy)
-                sparse_phase_a_kernel<T, K, false, false><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, ns, n_cg);
+                sparse_phase_a_kernel<T, K, false, false><<<g, kThreads, 0, s>>>(t, sg);
             else
-                sparse_phase_a_kernel<T, K, false, true><<<g, kThreads, 0, s>>>(t, (int)n_apply, (int)n_stream, ns, n_cg);
+                sparse_phase_a_kernel<T, K, false, true><<<g, kThreads, 0, s>>>(t, sg);
             cudaError_t e = cudaGetLastError();
             if (e != cudaSuccess) return e;
             phase_a = true;
@@ -1777,15 +1822,15 @@ static cudaError_t launch_sparse(const TransportArgs& t, cudaStream_t s) {
         cfg.numAttrs = 1;
         cudaError_t e;
         if (by_plane) {
-            if (vec && !copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, false, K>, t, n_cg);
-            else if (vec) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, true, K>, t, n_cg);
-            else if (!copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, false, K>, t, n_cg);
-            else e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, true, K>, t, n_cg);
+            if (vec && !copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, false, K>, t, sg);
+            else if (vec) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, true, K>, t, sg);
+            else if (!copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, false, K>, t, sg);
+            else e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, true, K>, t, sg);
         } else {
-            if (vec && !copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, false, 0>, t, n_cg);
-            else if (vec) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, true, 0>, t, n_cg);
-            else if (!copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, false, 0>, t, n_cg);
-            else e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, true, 0>, t, n_cg);
+            if (vec && !copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, false, 0>, t, sg);
+            else if (vec) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, true, true, 0>, t, sg);
+            else if (!copy) e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, false, 0>, t, sg);
+            else e = cudaLaunchKernelEx(&cfg, sparse_phase_b_kernel<T, false, true, 0>, t, sg);
         }
         if (e != cudaSuccess) return e;
     }
