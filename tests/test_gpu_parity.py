@@ -229,6 +229,36 @@ def test_ragged_tiles_and_many_views(gc):
     _run_step(gc, wv, g, oracle.rotate_anchors(64, 12, 1), synth.recon_params(wv, 0), mode="table")
 
 
+@pytest.mark.parametrize("seed", range(6))
+def test_random_shapes_split_the_grid_right(gc, seed):
+    # random (B, N, a, C, H, W): the step kernels split their block index into
+    # (asset, view, tile, channel group, record slice) with launch-invariant
+    # divisors; every shape must still equal the oracle, and the sparse step
+    # the mask-mode step bit for bit (both with and without the increment plane)
+    rng = np.random.default_rng(9000 + seed)
+    B, N = int(rng.integers(1, 4)), int(rng.integers(2, 11))
+    a, C = int(rng.integers(1, N)), int(rng.integers(1, 21))
+    H, W = int(rng.integers(7, 76)), int(rng.integers(7, 76))
+    cams = np.stack([synth.look_at_camera(az + 11.0 * seed, el, H, W)
+                     for az, el in synth.ring_layout(N, el_deg=10.0)]).astype(np.float32)
+    shapes = [synth.unit_sphere() if b % 2 == 0 else synth.random_solids(np.random.default_rng(seed * 10 + b))
+              for b in range(B)]
+    maps = [synth.render_asset(sh, cams, H, W) for sh in shapes]
+    w = synth.make_workload("tiny", H=H, W=W)
+    w = synth.Workload(**{**w.__dict__, "B": B, "N": N, "a": a, "C": C, "dtype": "bf16", "sampler": "ddim", "S": 30,
+                          "cams": np.ascontiguousarray(np.tile(cams[None], (B, 1, 1))),
+                          "pos": np.stack([m[0] for m in maps]), "valid": np.stack([m[1] for m in maps])})
+    g = DeviceGeometry(w, K=4, tables=False, source_index=False)
+    anchors = sorted(rng.choice(N, size=a, replace=False).tolist())
+    params = synth.recon_params(w, 7)
+    _, _, got_sparse, _ = _run_step(gc, w, g, anchors, params)
+    _, _, got_min, _ = _run_step(gc, w, g, anchors, params, minimal_ws=True)
+    _, _, got_mask, _ = _run_step(gc, w, g, anchors, params, mode="mask")
+    np.testing.assert_array_equal(got_sparse, got_mask)
+    np.testing.assert_array_equal(got_min, got_mask)
+    print("B=%d N=%d a=%d C=%d %dx%d anchors %s: %d records" % (B, N, a, C, H, W, anchors, g.n_records))
+
+
 def test_empty_asset_keeps_state(gc, workloads):
     # an asset with no foreground: tau = 0, no taps, every target keeps x0
     w = workloads("hunyuan64")
