@@ -182,6 +182,20 @@ def test_fm_velocity_and_k1(gc, workloads):
         _run_step(gc, w, g, [1, 3, 5], synth.recon_params(w, step), pred="velocity")
 
 
+@pytest.mark.parametrize("name,K,C,inplace", [("solids96", 1, 12, False), ("tiny", 4, 9, False),
+                                               ("tiny", 1, 16, True)])
+def test_plane_path_k1_and_f32(gc, workloads, name, K, C, inplace):
+    # the increment-plane path (C >= 8) with one tap per record and with f32
+    # latents: equal to the oracle, and bitwise to the record-parallel apply
+    w = workloads(name)
+    g = DeviceGeometry(w, K=K, tables=False, source_index=False)
+    anchors = [1, 3, 5] if w.N == 6 and w.a == 3 else [0, 3]
+    params = synth.recon_params(w, 1 if w.S > 1 else 0)
+    _, _, got_plane, _ = _run_step(gc, w, g, anchors, params, C=C, inplace=inplace)
+    _, _, got_rows, _ = _run_step(gc, w, g, anchors, params, C=C, inplace=inplace, minimal_ws=True)
+    np.testing.assert_array_equal(got_plane, got_rows)
+
+
 def test_in_place_cache_and_latents(gc, workloads):
     w = workloads("hunyuan64")
     g = DeviceGeometry(w, K=4, tables=False)
