@@ -890,8 +890,12 @@ def main():
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record()
+        # an NVTX range around the timed trajectories lets a profiler list
+        # exactly their launches (ncu --nvtx --nvtx-include "timed_trajectories/")
+        torch.cuda.nvtx.range_push("timed_trajectories")
         for _ in range(args.steps):
             launches += one_step(events)
+        torch.cuda.nvtx.range_pop()
         t1.record()
         torch.cuda.synchronize()
         barrier()
