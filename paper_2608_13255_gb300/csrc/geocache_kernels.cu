@@ -425,9 +425,13 @@ __global__ void __launch_bounds__(256, 8) fill_records_kernel(const float* __res
                                                            const int32_t* __restrict__ tile_ptr, int N, int H,
                                                            int W, int T, geocache_tap_record* __restrict__ rec,
                                                            long long max_records) {
-    const int tile = blockIdx.x, vu = blockIdx.y, b = blockIdx.z;
-    const int v = vu / N, u = vu % N;
-    if (u == v) return;  // diagonal pairs have no records
+    // blockIdx.y runs over the N (N - 1) off-diagonal pairs (diagonal pairs
+    // have no records): v = y / (N - 1), and u the (y mod (N - 1))-th view
+    // other than v
+    const int tile = blockIdx.x, b = blockIdx.z;
+    const int v = (int)blockIdx.y / (N - 1), up = (int)blockIdx.y - v * (N - 1);
+    const int u = up + (up >= v);
+    const int vu = v * N + u;
     const int HW = H * W;
     const int t = threadIdx.x;
     const size_t ti = ((size_t)b * N * N + vu) * T + tile;
@@ -495,7 +499,7 @@ __global__ void __launch_bounds__(256, 8) fill_records_kernel(const float* __res
 
 cudaError_t launch_fill_records(const geocache_corr& c, cudaStream_t s) {
     const int T = tiles_per_view(c.H, c.W);
-    dim3 grid(T, c.N * c.N, c.B);
+    dim3 grid(T, c.N * (c.N - 1), c.B);
     if (c.K == 4)
         fill_records_kernel<4><<<grid, 256, 0, s>>>(c.pos, c.cams, c.keep, c.tile_ptr, c.N, c.H, c.W, T, c.records,
                                                     c.max_records);
