@@ -56,8 +56,9 @@ struct TransportArgs {
 
 // The sparse step with wide latents (C >= kPlaneMinChannels) keeps the
 // anchors' increments as a plane [b][anchor slot][channel group][token] x 4
-// channels in the workspace, after room for max_records * C floats: it is
-// used when the workspace holds both (see geocache_transport_workspace).
+// channels at the start of the workspace.  It takes that path only when the
+// workspace holds max_records * C floats plus the plane, so that a minimal
+// workspace keeps the per-record rows (see geocache_transport_workspace).
 constexpr int kPlaneMinChannels = 8;
 inline long long plane_floats(long long B, long long a, int C, long long HW) {
     return B * a * (long long)((C + 3) / 4) * 4 * HW;

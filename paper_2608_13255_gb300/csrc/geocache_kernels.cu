@@ -1167,6 +1167,12 @@ __global__ void __launch_bounds__(kThreads) transport_simple_kernel(const Transp
 //    increments in anchor order (deterministic: the mean over covering
 //    anchors of Eq. 1 with the aggregation of Sec. 3.2; tokens without a
 //    record keep x0(t-1)), then stores and reconstructs every token.
+// Wide latents (C >= 8) with room in the workspace take another phase A:
+// the anchor views streamed while their increments are written once as a
+// plane (4 channels per 16-byte word), from which phase B forms each
+// record's increment itself (sparse_phase_a_plane_kernel below).  Without
+// that room, phase A applies the records per source tile when the corr has
+// a source index (sparse_phase_a_src_kernel), else record-parallel.
 
 // Streamed rows of the quad of tokens p0.. of view v of asset b, channel
 // group cg: x0 (the anchor's fresh x0 or x0(t-1)) and x_t.
@@ -1722,10 +1728,11 @@ __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_src
     }
 }
 
-// The source-tile apply is used for wide latents (at least kSrcMinChannels
-// channels), where the record-parallel apply's per-channel gathers dominate
-// phase A; with few channels it is slower (it reads the anchors' whole
-// x0(t-1) rows instead of the tapped tokens).
+// The source-tile apply serves wide latents (at least kSrcMinChannels
+// channels) whose workspace has no room for the increment plane, where the
+// record-parallel apply's per-channel gathers dominate phase A; with few
+// channels it is slower (it reads the anchors' whole x0(t-1) rows instead of
+// the tapped tokens).
 constexpr int kSrcMinChannels = 8;
 // Record-parallel apply: CTAs per (pair, channel group) sized for about this
 // many records each, from the mean records per ordered view pair.
