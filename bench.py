@@ -486,7 +486,7 @@ class Trajectory:
 
     def run(self, events=None):
         """Enqueue one trajectory eagerly; returns the number of kernels launched.
-        events: list receiving (start, end) CUDA events around each cached step."""
+        events: list receiving (start, end, 1) CUDA events around each cached step."""
         import torch
         gc, w = self.gc, self.w
         launches = 0
@@ -506,7 +506,7 @@ class Trajectory:
             launches += n
             if timed:
                 e1.record()
-                events.append((e0, e1))
+                events.append((e0, e1, 1))
         self.launches = launches
         return launches
 
@@ -532,6 +532,9 @@ class Trajectory:
             self.g_build = torch.cuda.CUDAGraph()
             with torch.cuda.graph(self.g_build):
                 self.gc.build_corr(self.corr)
+            # one graph per sampler step (the e2e path waits for each step's
+            # uploads), and one per run of consecutive steps of one kind (full
+            # or cached: the timed trajectories)
             self.g_steps = []
             cache = None
             for t in range(self.w.S):
@@ -539,26 +542,42 @@ class Trajectory:
                 with torch.cuda.graph(g):
                     cache, _ = self._step(t, cache)
                 self.g_steps.append(g)
+            self.g_runs = []
+            cache, t = None, 0
+            while t < self.w.S:
+                cached = t in self.anchor_x0
+                u = t
+                while u < self.w.S and (u in self.anchor_x0) == cached:
+                    u += 1
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g):
+                    for k in range(t, u):
+                        cache, _ = self._step(k, cache)
+                self.g_runs.append((g, cached, u - t))
+                t = u
             self.replay(None)
             torch.cuda.synchronize()
         except RuntimeError as exc:
             print("bench: CUDA graph capture failed (%s); timing eager launches" % exc, file=sys.stderr)
-            self.g_build = self.g_steps = None
+            self.g_build = self.g_steps = self.g_runs = None
             return False
         return True
 
     def replay(self, events=None):
+        """Replay one trajectory: the build, then each run of full or cached
+        steps.  events: list receiving (start, end, steps) CUDA events around
+        each run of cached steps."""
         import torch
         self.g_build.replay()
-        for t, g in enumerate(self.g_steps):
-            timed = events is not None and t in self.anchor_x0
+        for g, cached, n in self.g_runs:
+            timed = events is not None and cached
             if timed:
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 e0.record()
             g.replay()
             if timed:
                 e1.record()
-                events.append((e0, e1))
+                events.append((e0, e1, n))
 
     def run_e2e(self, host, graph=None):
         """One trajectory from pinned host inputs to a host copy of the final
@@ -864,9 +883,9 @@ def main():
             dist.barrier()
 
     # every kernel launch of a trajectory is captured once in CUDA graphs (one
-    # for the correspondence build, one per sampler step) and replayed, so
-    # launches cost no host time; events between the replays time each
-    # cached step's transport kernels
+    # for the correspondence build, one per run of consecutive full or cached
+    # sampler steps) and replayed, so launches cost no host time; events
+    # between the replays time each run of cached steps' transport kernels
     events = []
     use_graphs = traj.capture()
     launches_per_traj = traj.launches
@@ -900,12 +919,13 @@ def main():
         torch.cuda.synchronize()
         barrier()
     ms = reduce_max(t0.elapsed_time(t1), world)
-    kernel_ms = [a.elapsed_time(b) for a, b in events]
+    kernel_ms = [(a.elapsed_time(b), n) for a, b, n in events]
     ms_per_step = ms / args.steps
     total_pixels = traj.pixels * world
     value = job_value(traj.pixels, world, ms_per_step / 1e3)
 
-    k_avg_ms = sum(kernel_ms) / len(kernel_ms)
+    k_launches = sum(n for _, n in kernel_ms)
+    k_avg_ms = sum(ms for ms, _ in kernel_ms) / k_launches
     alg = step_bytes(w)
     achieved = alg / (k_avg_ms / 1e3) / 1e9
     peak, peak_src = measured_peak()
@@ -983,13 +1003,15 @@ def main():
                        ws_bytes / 1e6, L2_BYTES // 2 ** 20),
                    "step": "tau + correspondence build + %d-step trajectory (%d cached transport steps, %d full "
                            "steps)" % (w.S, traj.n_cached, w.S - traj.n_cached),
-                   "launch": "CUDA graphs (one per sampler step) replayed" if use_graphs else "eager"},
+                   "launch": ("CUDA graphs (the build; each run of consecutive full or cached sampler steps) "
+                              "replayed" if use_graphs else "eager")},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_source": peak_src,
                      "kernel": "sparse_phase_a_kernel + sparse_phase_b_kernel (one cached step)",
                      "alg_bytes_per_launch": alg,
-                     "avg_launch_us": 1e3 * k_avg_ms, "launches": len(kernel_ms),
-                     "timed_by": "events around each cached step's graph replay (launch included)",
+                     "avg_launch_us": 1e3 * k_avg_ms, "launches": k_launches,
+                     "timed_by": ("events around each graph replay of a run of consecutive cached steps "
+                                  "(graph launch included), divided by its steps"),
                      "frac_of_8TBs": achieved / 8000.0},
         "gpu_launches": launches,
         "pack_anchors": pack,
