@@ -116,7 +116,9 @@ typedef struct {
     const geocache_camera* cams;    /* device [B,N] */
     float* tau;                     /* device [B] f32, written by geocache_build_corr */
     int32_t* idx;                   /* device [B,N(v),N(u),H,W,K] i32 source token index row*W+col,
-                                       -1 = tap not kept; or NULL (tables not built) */
+                                       -1 = tap not kept; or NULL (tables not built).  A TABLE-mode
+                                       step drops an index outside [-1, H*W) and reports it through
+                                       the device status word (EINVAL) */
     float* w;                       /* device [B,N(v),N(u),H,W,K] f32 weights, 0 where idx = -1; or NULL */
     uint8_t* keep;                  /* device [B,N(v),N(u),H,W] u8: bit k set iff tap k is kept; or NULL */
     int32_t* tile_ptr;              /* device [B*N*N*T + 1] i32 (T = ceil(H*W / GEOCACHE_TILE_TOKENS)):
@@ -424,10 +426,12 @@ int geocache_rotate_anchors(int N, int a, int step, int S, const geocache_schedu
  * exceed max_records (the excess is dropped; transport steps read only the
  * records that exist), a record permutation entry out of range
  * (geocache_permute_records keeps that record), a mesh face with a vertex
- * index out of range (geocache_raster_posmaps skips it), and a bounded wait inside a
- * kernel that ran out (its CTA returns without writing its outputs).
+ * index out of range (geocache_raster_posmaps skips it), a correspondence
+ * table index outside [-1, H*W) in a TABLE-mode step (that tap is dropped),
+ * and a bounded wait inside a kernel that ran out (its CTA returns without
+ * writing its outputs).
  * Returns GEOCACHE_OK, ESHAPE (record overflow), EINVAL (bad permutation
- * entry or face index), ETIMEOUT (a wait gave up) or ECUDA.
+ * entry, face index or table index), ETIMEOUT (a wait gave up) or ECUDA.
  * ------------------------------------------------------------------------ */
 int geocache_device_status(void* stream);
 

@@ -130,6 +130,9 @@ int geocache_device_status(void* stream) {
     if (word & 8u)
         return fail(GEOCACHE_EINVAL, "a mesh face had a vertex index outside [0, n_verts) (status word 0x%x); "
                                      "those faces were skipped", word);
+    if (word & 16u)
+        return fail(GEOCACHE_EINVAL, "a correspondence table index was outside [-1, H*W) (status word 0x%x); "
+                                     "those taps were dropped", word);
     if (word) return fail(GEOCACHE_ETIMEOUT, "a bounded device wait gave up (status word 0x%x); outputs of that call are incomplete", word);
     return ok();
 }

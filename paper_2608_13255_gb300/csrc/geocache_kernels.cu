@@ -319,7 +319,8 @@ cudaError_t launch_build_corr(const geocache_corr& c, cudaStream_t s) {
 
 // Device status word (the library's only device-resident state): bit 0 = a
 // bounded wait gave up, bit 1 = the sparse form did not fit max_records,
-// bit 2 = a record permutation entry was out of range.
+// bit 2 = a record permutation entry was out of range, bit 4 = a table index
+// was outside [-1, H*W) (bit 3 is the rasteriser's word's bad face index).
 // Read and cleared by geocache_device_status().
 __device__ unsigned int g_device_error = 0;
 
@@ -800,9 +801,16 @@ __device__ __forceinline__ void item_taps(const TransportArgs& args, const geoca
         tp.kept = 0;
 #pragma unroll
         for (int kk = 0; kk < K; ++kk) {
-            tp.q[kk] = __ldg(args.idx + row * K + kk);
-            tp.w[kk] = __ldg(args.w + row * K + kk);
-            tp.kept += tp.q[kk] >= 0;
+            int q = __ldg(args.idx + row * K + kk);
+            float wq = __ldg(args.w + row * K + kk);
+            if (q < -1 || q >= (int)plane) {  // a caller's table with an index outside the view: dropped, reported
+                atomicOr(&g_device_error, 16u);
+                q = -1;
+                wq = 0.0f;
+            }
+            tp.q[kk] = q;
+            tp.w[kk] = wq;
+            tp.kept += q >= 0;
         }
         return;
     }

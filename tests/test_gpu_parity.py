@@ -427,6 +427,44 @@ def test_record_overflow_is_reported_not_faulted(gc, workloads):
     assert torch.isfinite(out).all()
 
 
+@pytest.mark.parametrize("name", ["hunyuan64", "ragged"])
+def test_table_index_out_of_range_is_dropped_and_reported(gc, workloads, name):
+    # a caller's correspondence table with indices outside the view (past the
+    # last token, and below -1): a TABLE-mode step drops those taps instead of
+    # reading outside the view, reports EINVAL through the device status word,
+    # and equals bit for bit the step on the same table with those taps
+    # removed (64 x 64: the staged kernel; 37 x 53: the per-tile kernel)
+    w = workloads("hunyuan64") if name == "hunyuan64" else synth.make_workload("batch128", B=1, H=37, W=53)
+    g = DeviceGeometry(w, K=4, tables=True)
+    torch.cuda.synchronize()
+    HW = w.H * w.W
+    idx, wt = g.idx.clone(), g.wt.clone()
+    kept = torch.nonzero(idx.view(-1) >= 0).view(-1)
+    bad = kept[torch.randperm(kept.numel(), generator=torch.Generator().manual_seed(4))[:64].cuda()]
+    idx.view(-1)[bad[:32]] = HW + 5
+    idx.view(-1)[bad[32:]] = -7
+    clean_idx, clean_wt = idx.clone(), wt.clone()
+    clean_idx.view(-1)[bad] = -1
+    clean_wt.view(-1)[bad] = 0.0
+    anchors = [0, 3]
+    x0_prev, x0_new, _ = step_inputs(w, 3, anchors)
+    d_prev, d_new = torch.from_numpy(x0_prev).cuda(), torch.from_numpy(x0_new).cuda()
+    outs = []
+    for ti, tw in ((idx, wt), (clean_idx, clean_wt)):
+        c = gc.make_corr(g.pos, g.valid, g.cams, g.tau, ti, tw, K=4, tol_frac=w.tol_frac, mode=gc.CORR_TABLE)
+        out = torch.empty_like(d_prev)
+        gc.transport_step(c, anchors, w.C, d_new, d_prev, out)
+        torch.cuda.synchronize()
+        outs.append(out)
+        if ti is idx:
+            with pytest.raises(gc.GeocacheError) as ei:
+                gc.device_status()
+            assert ei.value.status == gc.EINVAL and "table index" in str(ei.value)
+        gc.device_status()  # clean
+    assert torch.isfinite(outs[0]).all()
+    assert torch.equal(outs[0].view(torch.int32), outs[1].view(torch.int32))
+
+
 def test_graph_replay_matches_eager(gc, workloads):
     # a cached step captured in a CUDA graph (with the programmatic
     # dependency between its two kernels) gives the eager results
