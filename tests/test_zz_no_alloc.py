@@ -68,6 +68,24 @@ def test_noalloc_matches_workspace_entry_point_on_consecutive_calls(gc, sampler,
         assert np.abs(got_x0.numpy() - x0_prev).max() > 1e-3
 
 
+def test_noalloc_wide_latents_match_the_plane_path(gc):
+    # ring12_128 (C = 16): the built-in array holds max_records * C floats but
+    # not the anchors' increment plane as well, so the no-alloc step applies
+    # the records into rows while the workspace entry point (sized by
+    # geocache_transport_workspace) takes the plane; the bits must agree
+    w = synth.make_workload("ring12_128")
+    g = DeviceGeometry(w, K=4, tables=False, source_index=False)
+    need = g.corr.min_workspace_floats(w.C)
+    plane = w.B * w.a * 4 * (-(-w.C // 4)) * w.H * w.W
+    assert need <= 4 * 1024 * 1024 < need + plane
+    for anchors, step in (([0, 3, 6, 9], 2), ([1, 4, 7, 10], 3)):
+        for in_place in (False, True):
+            ref_x0, ref_xn, _ = _step(gc, g, w, anchors, step, noalloc=False, in_place=in_place)
+            got_x0, got_xn, _ = _step(gc, g, w, anchors, step, noalloc=True, in_place=in_place)
+            assert torch.equal(got_x0.view(torch.int32), ref_x0.view(torch.int32))
+            assert torch.equal(got_xn.view(torch.int16), ref_xn.view(torch.int16))
+
+
 def test_noalloc_rejects_steps_beyond_its_scratch(gc):
     # a sparse-mode step whose scratch (max_records * C floats) exceeds the
     # built-in array is refused before any launch
