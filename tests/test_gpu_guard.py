@@ -140,12 +140,14 @@ def test_transport_writes_only_its_outputs(gc, case):
             d_xt.check("%s %s in place: x_t" % (case, mode))
 
 
-@pytest.mark.parametrize("frac", [1.0, 0.5])
-def test_record_buffer_at_and_beyond_capacity(gc, frac):
+@pytest.mark.parametrize("frac,C", [(1.0, 4), (0.5, 4), (1.0, 16), (0.5, 16)])
+def test_record_buffer_at_and_beyond_capacity(gc, frac, C):
     # records filled exactly to max_records, and an overflowing build (half
     # the capacity needed): nothing is written past the buffer, the overflow
     # is reported, and a step over the truncated form stays inside its outputs
+    # (C = 16: the increment-plane path)
     w = synth.make_workload("batch128", B=2, H=37, W=53)
+    w = synth.Workload(**{**w.__dict__, "C": C})
     corr, g, R, cap, _ = _geometry(gc, w, K=4)
     if frac < 1.0:
         corr, g, R, cap, _ = _geometry(gc, w, K=4, records_frac=frac)
