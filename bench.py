@@ -735,13 +735,14 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
-def measured_traffic(kernel_hash, assets):
-    """DRAM bytes of one transport step from the committed ncu summary,
-    scaled to `assets`; None when the kernels changed since the capture."""
+def measured_traffic(kernel_hash, assets, workload):
+    """DRAM bytes of one transport step from the committed ncu summary of
+    `workload`, scaled to `assets`; None when the kernels changed since the
+    capture or no summary covers the workload."""
     path = os.path.join(ROOT, "profiles", "transport_traffic.txt")
     try:
         kv = dict(line.split() for line in open(path) if line.strip() and not line.startswith("#"))
-        if kv.get("kernel_hash") != kernel_hash:
+        if kv.get("kernel_hash") != kernel_hash or kv.get("workload") != workload:
             return None
         return float(kv["bytes_per_step"]) * assets / float(kv["assets"])
     except (OSError, ValueError, KeyError):
@@ -958,7 +959,7 @@ def main():
     alg = step_bytes(w)
     achieved = alg / (k_avg_ms / 1e3) / 1e9
     peak, peak_src = measured_peak()
-    traffic = measured_traffic(gbuild.source_hash(), w.B)
+    traffic = measured_traffic(gbuild.source_hash(), w.B, w.name)
 
     # secondary: anchor-row pack of the latents and scatter back (the batch
     # slicing around the denoiser's anchor-only forward); four source / slice
