@@ -61,10 +61,21 @@ def is_stale() -> bool:
 
 
 def build(force: bool = False, verbose: bool = False, extra_flags=()) -> str:
-    """Compile and link libgeocache.so if any source changed; return its path."""
+    """Compile and link libgeocache.so if any source changed; return its path.
+    Processes that build at the same time (one per rank) take turns on a lock
+    file, so that none links objects another is still writing."""
     if not force and not is_stale():
         return LIB
+    import fcntl
     os.makedirs(LIBDIR, exist_ok=True)
+    with open(os.path.join(LIBDIR, ".build.lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        if not force and not is_stale():  # another process built it meanwhile
+            return LIB
+        return _build_locked(verbose, extra_flags)
+
+
+def _build_locked(verbose, extra_flags) -> str:
     cc = nvcc()
     objs, procs = [], []
     for src in _sources():
