@@ -1433,11 +1433,13 @@ template <typename T>
 constexpr int kPhaseABlocks = sizeof(T) == 2 ? 6 : 1;
 template <typename T>
 constexpr int kPhaseBBlocks = sizeof(T) == 2 ? 5 : 1;
-// The increment-plane kernels (wide latents) at 4 resident CTAs per SM: no
-// spills (62 / 64 registers); at 5 or 6 the spills cost more than the
-// residency gains.
+// The increment-plane kernels (wide latents): phase A at 4 resident CTAs per
+// SM (62 registers; at 5 or 6 its spills cost more than the residency
+// gains), phase B at 5 (46 registers, no spills: it loads its streamed rows
+// after the fold, so they are not held across the gathers; 4 or 6 resident
+// CTAs, or the rows prefetched into the L2 before the wait, were slower).
 constexpr int kPlaneABlocks = 4;
-constexpr int kPlaneBBlocks = 4;
+constexpr int kPlaneBBlocks = 5;
 
 template <typename T, int K, bool VEC, bool COPY>
 __global__ void __launch_bounds__(kThreads, kPhaseABlocks<T>) sparse_phase_a_kernel(const TransportArgs args,
@@ -1509,9 +1511,11 @@ __global__ void __launch_bounds__(kThreads, PK ? kPlaneBBlocks : kPhaseBBlocks<T
         return;
     }
     const int v = args.others[blockIdx.y];
-    // streamed rows first (phase A writes none of them), tile offsets next
+    // streamed rows first (phase A writes none of them), tile offsets next;
+    // with the plane (PK) the rows are loaded after the fold instead, which
+    // keeps the fold's registers free for more resident CTAs
     QuadRows<T, VEC> q;
-    if (cnt > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
+    if (!PK && cnt > 0) q.load(args, b, v, -1, p0, cnt, cg, cn);
     if (t < a) {
         const size_t i = (((size_t)b * N + v) * N + args.anchors[t]) * T_tiles + tile;
         // ranges clamped to the records that exist (an overflow is reported by the build)
@@ -1533,12 +1537,18 @@ __global__ void __launch_bounds__(kThreads, PK ? kPlaneBBlocks : kPhaseBBlocks<T
     // completes only after phase A
     const bool first = blockIdx.x == 0 && blockIdx.y == 0 && blockIdx.z == 0;
     if (total == 0 && !first) {
-        if (cnt > 0) q.store(args, b, v, p0, cnt, cg, cn);
+        if (cnt > 0) {
+            if (PK) q.load(args, b, v, -1, p0, cnt, cg, cn);
+            q.store(args, b, v, p0, cnt, cg, cn);
+        }
         return;
     }
     pdl_wait();  // phase A's workspace writes are complete and visible
     if (total == 0) {  // no record in the tile: every token keeps x0(t-1), nothing to fold
-        if (cnt > 0) q.store(args, b, v, p0, cnt, cg, cn);
+        if (cnt > 0) {
+            if (PK) q.load(args, b, v, -1, p0, cnt, cg, cn);
+            q.store(args, b, v, p0, cnt, cg, cn);
+        }
         return;
     }
     for (int j0 = 0; j0 < total; j0 += kThreads) {
@@ -1605,6 +1615,7 @@ __global__ void __launch_bounds__(kThreads, PK ? kPlaneBBlocks : kPhaseBBlocks<T
         }
     }
     if (cnt > 0) {
+        if (PK) q.load(args, b, v, -1, p0, cnt, cg, cn);
         const uint32_t n4 = *reinterpret_cast<const uint32_t*>(s_n + 4 * t);
         if (n4) q.template fold4<COPY>(s_acc, n4, 4 * t);
         q.store(args, b, v, p0, cnt, cg, cn);
