@@ -61,8 +61,8 @@ __device__ __forceinline__ float fold_one(bool copy, float x0, float g, int n) {
 
 // -------------------------------------------------------------------- tau --
 // One thread-block cluster per asset: CTA r of the cluster reduces the
-// componentwise min / max of the foreground texels of views r, r + CS, ...
-// (exact and order-free), the cluster combines the partial boxes through
+// componentwise min / max of the foreground texels of slice r of the asset's
+// texels (exact and order-free), the cluster combines the partial boxes through
 // distributed shared memory, and CTA 0 writes tau = tol_frac * sqrt(diag^2)
 // with the squares summed ((d0^2 + d1^2) + d2^2) in binary32.
 struct Box {
@@ -82,8 +82,8 @@ __device__ __forceinline__ void box_reduce_warp(Box& x) {
     }
 }
 
-__global__ void __launch_bounds__(512) tau_kernel(const float* __restrict__ pos, const uint8_t* __restrict__ valid,
-                                                  int N, int HW, float tol_frac, int quads, float* __restrict__ tau) {
+__global__ void __launch_bounds__(256, 8) tau_kernel(const float* __restrict__ pos, const uint8_t* __restrict__ valid,
+                                                     int N, int HW, float tol_frac, int quads, float* __restrict__ tau) {
     namespace cg = cooperative_groups;
     cg::cluster_group cluster = cg::this_cluster();
     const int cs = (int)cluster.num_blocks();
@@ -95,38 +95,43 @@ __global__ void __launch_bounds__(512) tau_kernel(const float* __restrict__ pos,
 #pragma unroll
     for (int c = 0; c < 3; ++c) { x.lo[c] = FLT_MAX; x.hi[c] = -FLT_MAX; }
     x.any = 0;
-    for (int v = rank; v < N; v += cs) {
-        const size_t base = ((size_t)b * N + v) * HW;
-        if (quads) {  // four texels per load: their 4 validity bytes and 12 position floats
-            const uint32_t* vq = reinterpret_cast<const uint32_t*>(valid + base);
-            const float4* pq = reinterpret_cast<const float4*>(pos + 3 * base);
+    // the asset's N views are contiguous: each CTA of the cluster takes one
+    // slice of their N * HW texels
+    const size_t n = (size_t)N * HW;
+    const size_t base = (size_t)b * n;
+    if (quads) {  // four texels per load: their 4 validity bytes and 12 position floats
+        const size_t nq = n / 4, per = (nq + cs - 1) / cs;
+        const size_t q0 = (size_t)rank * per, q1 = q0 + per < nq ? q0 + per : nq;
+        const uint32_t* vq = reinterpret_cast<const uint32_t*>(valid + base);
+        const float4* pq = reinterpret_cast<const float4*>(pos + 3 * base);
 #pragma unroll 4
-            for (int i = threadIdx.x; i < HW / 4; i += blockDim.x) {
-                const uint32_t m = __ldg(vq + i);
-                if (!m) continue;
-                x.any = 1;
-                const float4 f0 = __ldg(pq + 3 * i), f1 = __ldg(pq + 3 * i + 1), f2 = __ldg(pq + 3 * i + 2);
-                const float f[12] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w, f2.x, f2.y, f2.z, f2.w};
+        for (size_t i = q0 + threadIdx.x; i < q1; i += blockDim.x) {
+            const uint32_t m = __ldg(vq + i);
+            if (!m) continue;  // background quads: their positions are not read
+            x.any = 1;
+            const float4 f0 = __ldg(pq + 3 * i), f1 = __ldg(pq + 3 * i + 1), f2 = __ldg(pq + 3 * i + 2);
+            const float f[12] = {f0.x, f0.y, f0.z, f0.w, f1.x, f1.y, f1.z, f1.w, f2.x, f2.y, f2.z, f2.w};
 #pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    if (!((m >> (8 * k)) & 0xffu)) continue;
-#pragma unroll
-                    for (int c = 0; c < 3; ++c) {
-                        x.lo[c] = fminf(x.lo[c], f[3 * k + c]);
-                        x.hi[c] = fmaxf(x.hi[c], f[3 * k + c]);
-                    }
-                }
-            }
-        } else {
-            for (int i = threadIdx.x; i < HW; i += blockDim.x) {
-                if (!__ldg(valid + base + i)) continue;
-                x.any = 1;
+            for (int k = 0; k < 4; ++k) {
+                if (!((m >> (8 * k)) & 0xffu)) continue;
 #pragma unroll
                 for (int c = 0; c < 3; ++c) {
-                    const float p = __ldg(pos + 3 * (base + i) + c);
-                    x.lo[c] = fminf(x.lo[c], p);
-                    x.hi[c] = fmaxf(x.hi[c], p);
+                    x.lo[c] = fminf(x.lo[c], f[3 * k + c]);
+                    x.hi[c] = fmaxf(x.hi[c], f[3 * k + c]);
                 }
+            }
+        }
+    } else {
+        const size_t per = (n + cs - 1) / cs;
+        const size_t i0 = (size_t)rank * per, i1 = i0 + per < n ? i0 + per : n;
+        for (size_t i = i0 + threadIdx.x; i < i1; i += blockDim.x) {
+            if (!__ldg(valid + base + i)) continue;
+            x.any = 1;
+#pragma unroll
+            for (int c = 0; c < 3; ++c) {
+                const float p = __ldg(pos + 3 * (base + i) + c);
+                x.lo[c] = fminf(x.lo[c], p);
+                x.hi[c] = fmaxf(x.hi[c], p);
             }
         }
     }
@@ -171,10 +176,13 @@ __global__ void __launch_bounds__(512) tau_kernel(const float* __restrict__ pos,
 
 cudaError_t launch_tau(const float* pos, const uint8_t* valid, int B, int N, int H, int W, float tol_frac,
                        float* tau, cudaStream_t s) {
-    const int cs = N < 8 ? N : 8;  // portable cluster size
+    // a cluster of 8 CTAs (the portable size) per asset: 1024 CTAs for 128
+    // assets, resident at once at 8 per SM (one CTA per view at 512 threads,
+    // 768 CTAs in 1.3 waves, took 16 us more per 128-asset build)
+    const int cs = 8;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(B * cs);
-    cfg.blockDim = dim3(512);
+    cfg.blockDim = dim3(256);
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
