@@ -451,6 +451,23 @@ def measure_supersampled(dev, B=16, H=128, W=128, s=4, reps=5):
             "pooled_equals_fused": same}
 
 
+def step_runs(S, cached_steps):
+    """The graphs of one trajectory: (first step, end step, cached, head) per
+    run of consecutive sampler steps of one kind, in order.  head marks a run
+    of full steps that opens the trajectory: full steps read no
+    correspondence, so the build runs beside them on a side stream of the same
+    graph, joined before the first cached step."""
+    runs, t = [], 0
+    while t < S:
+        cached = t in cached_steps
+        u = t
+        while u < S and (u in cached_steps) == cached:
+            u += 1
+        runs.append((t, u, cached, t == 0 and not cached))
+        t = u
+    return runs
+
+
 class Trajectory:
     """Device state of one batch's trajectory and the loop over its steps."""
 
@@ -574,16 +591,8 @@ class Trajectory:
             self.g_runs = []
             self.build_in_head = False
             side = torch.cuda.Stream()
-            cache, t = None, 0
-            while t < self.w.S:
-                cached = t in self.anchor_x0
-                u = t
-                while u < self.w.S and (u in self.anchor_x0) == cached:
-                    u += 1
-                # a trajectory that opens with full steps (they read no
-                # correspondence) runs the build beside them, on a side stream
-                # of the same graph joined before the first cached step
-                head = t == 0 and not cached
+            cache = None
+            for t, u, cached, head in step_runs(self.w.S, set(self.anchor_x0)):
                 g = torch.cuda.CUDAGraph()
                 with torch.cuda.graph(g):
                     if head:
@@ -597,7 +606,6 @@ class Trajectory:
                         cur.wait_stream(side)
                 self.build_in_head = self.build_in_head or head
                 self.g_runs.append((g, cached, u - t))
-                t = u
             self.replay(None)
             torch.cuda.synchronize()
         except RuntimeError as exc:

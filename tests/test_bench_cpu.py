@@ -53,3 +53,23 @@ def test_reference_arm_prints_one_json_line():
     assert d["value"] > 0 and d["higher_is_better"] is True and d["steps"] == 1
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
+
+
+@pytest.mark.parametrize("name", ["batch128", "hunyuan64", "solids96", "ring12_128", "tiny"])
+def test_step_runs_cover_the_trajectory(name):
+    """The bench's graphs: maximal runs of one kind of step, in order, covering
+    every sampler step once; the build joins the first run exactly when the
+    trajectory opens with a full step (the schedule from the oracle)."""
+    import oracle
+    w = synth.make_workload(name, B=1)
+    cached = {t for t in range(w.S) if not oracle.is_full_step(t, w.S, w.schedule)}
+    runs = bench.step_runs(w.S, cached)
+    assert runs[0][0] == 0 and runs[-1][1] == w.S
+    for (t0, u0, c0, _), (t1, u1, c1, _) in zip(runs, runs[1:]):
+        assert u0 == t1 and c0 != c1
+    for t, u, c, head in runs:
+        assert t < u and all((k in cached) == c for k in range(t, u))
+        assert head == (t == 0 and not c)
+    assert runs[0][3] == (0 not in cached)
+    if name == "batch128":  # a full step every fifth step: F CCCC x 6
+        assert [(u - t, c) for t, u, c, _ in runs] == [(1, False), (4, True)] * 6
